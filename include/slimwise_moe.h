@@ -1,0 +1,190 @@
+/*
+ * slimwise_moe.h -- C ABI of the GB300 (sm_103a) pruned-pool batched-decode
+ * MoE layer.
+ *
+ * The layer is the decode-phase MoE block of SlimWise (arXiv 2609.34117):
+ * decode runs over a retained expert set K' of m' experts out of m, selected
+ * by masking the router (Sec. 3.1, Eq. 2); the top-k (k unchanged by pruning,
+ * Sec. 2.3) gates are renormalised over the k selected experts alone
+ * (Sec. 3.1); each step streams only the weights of the union of experts
+ * selected across the batch (Sec. 2.1, Eq. 1).  For every token t:
+ *
+ *   z[t,e]   = x_t . Wr[e]                          e in K'
+ *   S_t      = top-k of z[t, K'] (logit desc, id asc on ties)
+ *   g[t,j]   = exp(z_j - z_1) / sum_{j' in S_t} exp(z_j' - z_1)
+ *   y_e(x)   = W_down[e] (SiLU(W_gate[e] x) * (W_up[e] x))
+ *   out[t]   = sum_{j=0..k-1} g[t,j] y_{S_t[j]}(x_t)
+ *
+ * Conventions shared by every entry point
+ *   - All array arguments are DEVICE pointers owned by the caller; the
+ *     library never allocates, frees or retains them after returning.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and the call returns without synchronising.  Calls that share a
+ *     workspace must be ordered (same stream, or synchronised): the workspace
+ *     holds the routing state and the intermediate activations of one call.
+ *   - Errors are returned as a slimwise_status value; nothing is enqueued
+ *     when a host-side check fails.  A device-side wait that timed out is
+ *     reported by slimwise_moe_device_status().
+ *   - Layouts are row-major; bf16 is IEEE bfloat16 stored in 16 bits.
+ *   - Every pointer must be 16-byte aligned.
+ *   - Supported shapes: H % 128 == 0, I % 64 == 0, 1 <= E <= 1024,
+ *     1 <= top_k <= min(32, m'), B >= 0 (B == 0 is a no-op).
+ */
+#ifndef SLIMWISE_MOE_H_
+#define SLIMWISE_MOE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum slimwise_status {
+  SLIMWISE_OK = 0,
+  SLIMWISE_ERR_INVALID_ARG = 1,       /* null pointer, k / m' / B out of range */
+  SLIMWISE_ERR_UNSUPPORTED_SHAPE = 2, /* H, I, E or alignment not supported     */
+  SLIMWISE_ERR_WORKSPACE = 3,         /* workspace smaller than required        */
+  SLIMWISE_ERR_CUDA = 4,              /* a CUDA runtime call or launch failed   */
+  SLIMWISE_ERR_DEVICE = 5             /* a kernel reported a timeout / bad input */
+} slimwise_status;
+
+/* Device-side error bits reported by slimwise_moe_device_status(). */
+#define SLIMWISE_DEVERR_PIPELINE_TIMEOUT 0x1   /* an mbarrier wait gave up        */
+#define SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT 0x2 /* gate/up -> down wait gave up    */
+#define SLIMWISE_DEVERR_DUPLICATE_RETAINED 0x4 /* retained_idx has a repeated id  */
+#define SLIMWISE_DEVERR_BAD_RETAINED 0x8       /* retained_idx has an id outside [0,E) */
+#define SLIMWISE_DEVERR_BAD_TOPK 0x10          /* a given top-k id outside [0,E)  */
+
+/* Problem shape. */
+typedef struct slimwise_moe_shape {
+  int32_t num_tokens;  /* B: decode batch (tokens)           */
+  int32_t hidden;      /* H: model width                     */
+  int32_t num_experts; /* E: routed experts in the full pool */
+  int32_t inter;       /* I: expert intermediate width       */
+} slimwise_moe_shape;
+
+/* Human-readable name of a status code (static storage). */
+const char *slimwise_status_string(int status);
+
+/*
+ * Bytes of device workspace a call with this shape and top_k needs
+ * (routing state, grouped activations, expert outputs, counters).
+ * Returns SLIMWISE_OK and writes *bytes, or an error for an unsupported
+ * shape.  The workspace needs no initialisation and may be reused by
+ * consecutive calls on one stream.
+ */
+int slimwise_moe_workspace_size(const slimwise_moe_shape *shape, int32_t top_k,
+                                size_t *bytes);
+
+/*
+ * The decode MoE layer over the retained pool K' (Sec. 3.1, Eq. 2).
+ *
+ *   hidden       bf16 [B, H]     token hidden states
+ *   router_w     fp32 [E, H]     router weight of the full pool
+ *   retained_idx int32 [m']      ids of K', unique, in [0, E), any order
+ *                                (duplicates or out-of-range ids set a
+ *                                device error bit; results are then undefined)
+ *   n_retained   m', top_k <= m' <= E
+ *   w_gate_up    bf16 [E, 2I, H] rows [0, I) = gate, rows [I, 2I) = up
+ *   w_down       bf16 [E, H, I]
+ *   top_k        k, 1 <= k <= min(32, m')
+ *   out          bf16 [B, H]     gate-weighted sum of the k expert outputs
+ *   stream       cudaStream_t
+ *   workspace    >= slimwise_moe_workspace_size() bytes, 256-byte aligned
+ *
+ * Only the weights of experts selected by at least one token are read.
+ */
+int slimwise_moe_decode(const void *hidden, const float *router_w,
+                        const int32_t *retained_idx, int32_t n_retained,
+                        const void *w_gate_up, const void *w_down,
+                        int32_t top_k, void *out, void *stream,
+                        const slimwise_moe_shape *shape, void *workspace,
+                        size_t workspace_bytes);
+
+/*
+ * Full-pool variant: K' = all E experts (the unpruned layer that prefill runs,
+ * Sec. 3.1 "masking applied to neither phase").  Arguments as above.
+ */
+int slimwise_moe_decode_full(const void *hidden, const float *router_w,
+                             const void *w_gate_up, const void *w_down,
+                             int32_t top_k, void *out, void *stream,
+                             const slimwise_moe_shape *shape, void *workspace,
+                             size_t workspace_bytes);
+
+/*
+ * Launch options for slimwise_moe_decode_ex (all fields may be zero).
+ *   ffn_begin / ffn_end  cudaEvent_t recorded on `stream` immediately before
+ *                        and after the expert-FFN kernel (NULL: none); used to
+ *                        time that kernel alone.
+ *   disable_pdl          1: launch the three kernels with plain stream
+ *                        ordering instead of programmatic dependent launch.
+ *   grid_ctas            >0: persistent expert-FFN grid size (default: the
+ *                        device's SM count).
+ */
+typedef struct slimwise_decode_opts {
+  void *ffn_begin;
+  void *ffn_end;
+  int32_t disable_pdl;
+  int32_t grid_ctas;
+} slimwise_decode_opts;
+
+/* slimwise_moe_decode with launch options; retained_idx NULL = full pool. */
+int slimwise_moe_decode_ex(const void *hidden, const float *router_w,
+                           const int32_t *retained_idx, int32_t n_retained,
+                           const void *w_gate_up, const void *w_down,
+                           int32_t top_k, void *out, void *stream,
+                           const slimwise_moe_shape *shape, void *workspace,
+                           size_t workspace_bytes,
+                           const slimwise_decode_opts *opts);
+
+/*
+ * Routing only (Sec. 3.1: Eq. 2 mask, top-k, renormalised gates) followed by
+ * the grouping of slots by expert, with the results copied out (device
+ * buffers; any output may be NULL to skip it):
+ *   topk_idx   int32 [B, k]  selected expert ids, selection order
+ *   topk_gate  fp32  [B, k]  renormalised gates
+ *   counts     int32 [E]     slots routed to each expert
+ *   offsets    int32 [E+1]   exclusive prefix sum of counts
+ *   union_ids  int32 [E]     selected experts ascending, then -1 padding
+ *   union_size int32 [1]     number of distinct selected experts (Eq. 1)
+ *   perm       int32 [B*k]   flat slot t*k+j at grouped position p,
+ *                            ordered by (expert asc, token asc)
+ *   pos        int32 [B*k]   inverse of perm
+ * retained_idx NULL = full pool.
+ */
+int slimwise_moe_route(const void *hidden, const float *router_w,
+                       const int32_t *retained_idx, int32_t n_retained,
+                       int32_t top_k, void *stream,
+                       const slimwise_moe_shape *shape, void *workspace,
+                       size_t workspace_bytes, int32_t *topk_idx,
+                       float *topk_gate, int32_t *counts, int32_t *offsets,
+                       int32_t *union_ids, int32_t *union_size, int32_t *perm,
+                       int32_t *pos);
+
+/*
+ * Grouping of caller-given selections (the permutation stage alone), e.g. to
+ * measure union sizes for uniformly random selections against Eq. 1.
+ *   topk_idx  int32 [B, k] device; each row must hold k distinct ids in [0,E)
+ * Outputs as in slimwise_moe_route (any may be NULL).  Uses the workspace of
+ * shape {B, shape->hidden, E, shape->inter}.
+ */
+int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
+                       const slimwise_moe_shape *shape, void *workspace,
+                       size_t workspace_bytes, int32_t *counts,
+                       int32_t *offsets, int32_t *union_ids,
+                       int32_t *union_size, int32_t *perm, int32_t *pos);
+
+/*
+ * Reads (and synchronises `stream` for) the device error bits the last call
+ * on this workspace left (SLIMWISE_DEVERR_*), writing them to *flags.
+ * Returns SLIMWISE_OK if none are set, SLIMWISE_ERR_DEVICE otherwise.
+ */
+int slimwise_moe_device_status(const void *workspace, void *stream,
+                               int32_t *flags);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SLIMWISE_MOE_H_ */

@@ -1,0 +1,342 @@
+// common.cuh -- shared definitions of the sm_103a decode-MoE kernels:
+// workspace layout, kernel parameter blocks, and thin inline-PTX wrappers for
+// mbarrier, TMA (cp.async.bulk.tensor), tcgen05 (MMA / TMEM) and
+// programmatic dependent launch.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "slimwise_moe.h"
+
+namespace slimwise {
+
+// ---------------------------------------------------------------------------
+// Tiling constants of the expert-FFN kernel.
+// ---------------------------------------------------------------------------
+constexpr int kBlockK = 64;          // K elements per pipeline stage (128 B of bf16)
+constexpr int kTileRows = 128;       // MMA M: weight rows per work item
+constexpr int kGateRows = 64;        // gate rows (and as many up rows) per gate/up item
+constexpr int kMaxTokTile = 256;     // MMA N limit: tokens of one expert per item
+constexpr int kTokBox = 16;          // TMA box height for token rows
+constexpr int kATileBytes = kTileRows * kBlockK * 2;   // 16 KiB
+constexpr int kMaxExperts = 1024;
+constexpr int kMaxTopK = 32;
+constexpr int kCombineTile = 128;    // h values per down item (= kTileRows)
+
+// Tokens of one expert handled by one work item: the MMA N of the FFN
+// kernel, a multiple of 16 that covers the largest possible per-expert count
+// (B) up to the 256 limit.
+__host__ __device__ inline int token_chunk_for(int B) {
+  int c = (B + 15) / 16 * 16;
+  return c < 16 ? 16 : (c > kMaxTokTile ? kMaxTokTile : c);
+}
+
+// Control words at the head of the workspace (int32 each).
+enum CtrlWord {
+  kCtrlUnionSize = 0,
+  kCtrlNumEntries = 1,
+  kCtrlItems1 = 2,      // gate/up work items
+  kCtrlTotalItems = 3,  // gate/up + down work items
+  kCtrlWorkCounter = 4, // dynamic scheduler counter
+  kCtrlErr = 5,         // SLIMWISE_DEVERR_* bits of the current call
+  kCtrlWords = 16
+};
+
+// Byte offsets of every workspace region (all 1024-byte aligned).
+struct WsLayout {
+  size_t ctrl, topk_idx, topk_gate, counts, offsets, union_ids, entries,
+      entry_done, perm, pos, comb_cnt, xp, act, y, total;
+  int32_t max_entries;
+};
+
+__host__ __device__ inline size_t align_up(size_t v, size_t a) {
+  return (v + a - 1) / a * a;
+}
+
+inline WsLayout make_layout(int B, int H, int E, int I, int k) {
+  WsLayout L;
+  size_t o = 0;
+  const size_t slots = (size_t)B * k;
+  auto take = [&](size_t bytes) {
+    size_t r = o;
+    o = align_up(o + (bytes ? bytes : 1), 1024);
+    return r;
+  };
+  const size_t chunk = (size_t)token_chunk_for(B);
+  L.max_entries = E + (int32_t)((slots + chunk - 1) / chunk);
+  L.ctrl = take(kCtrlWords * 4);
+  L.topk_idx = take(slots * 4);
+  L.topk_gate = take(slots * 4);
+  L.counts = take((size_t)E * 4);
+  L.offsets = take((size_t)(E + 1) * 4);
+  L.union_ids = take((size_t)E * 4);
+  L.entries = take((size_t)L.max_entries * 16);
+  L.entry_done = take((size_t)L.max_entries * 4);
+  L.perm = take(slots * 4);
+  L.pos = take(slots * 4);
+  L.comb_cnt = take((size_t)B * (H / kCombineTile) * 4);
+  L.xp = take(slots * H * 2);
+  L.act = take(slots * I * 2);
+  L.y = take(slots * H * 4);
+  L.total = o;
+  return L;
+}
+
+// Device view of the workspace.
+struct Ws {
+  int32_t *ctrl;
+  int32_t *topk_idx;
+  float *topk_gate;
+  int32_t *counts;
+  int32_t *offsets;
+  int32_t *union_ids;
+  int4 *entries;       // {expert, slot_base, n_tokens, 0}
+  int32_t *entry_done; // gate/up items finished per entry
+  int32_t *perm;
+  int32_t *pos;
+  int32_t *comb_cnt;   // [B, H/128] down items finished per (token, h tile)
+  __nv_bfloat16 *xp;   // [B*k, H] hidden rows in grouped order
+  __nv_bfloat16 *act;  // [B*k, I] SwiGLU activations in grouped order
+  float *y;            // [B*k, H] expert outputs in grouped order
+};
+
+inline Ws make_ws(void *base, const WsLayout &L) {
+  char *b = (char *)base;
+  Ws w;
+  w.ctrl = (int32_t *)(b + L.ctrl);
+  w.topk_idx = (int32_t *)(b + L.topk_idx);
+  w.topk_gate = (float *)(b + L.topk_gate);
+  w.counts = (int32_t *)(b + L.counts);
+  w.offsets = (int32_t *)(b + L.offsets);
+  w.union_ids = (int32_t *)(b + L.union_ids);
+  w.entries = (int4 *)(b + L.entries);
+  w.entry_done = (int32_t *)(b + L.entry_done);
+  w.perm = (int32_t *)(b + L.perm);
+  w.pos = (int32_t *)(b + L.pos);
+  w.comb_cnt = (int32_t *)(b + L.comb_cnt);
+  w.xp = (__nv_bfloat16 *)(b + L.xp);
+  w.act = (__nv_bfloat16 *)(b + L.act);
+  w.y = (float *)(b + L.y);
+  return w;
+}
+
+struct Dims {
+  int B, H, E, I, k;
+  int m_ret;      // retained experts (E for the full pool)
+  int tok_chunk;  // max tokens of one expert per work item (multiple of 16, <= 256)
+};
+
+// Kernel launch declarations (defined in their own translation units).
+cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
+                              const int32_t *retained, Dims d, Ws ws,
+                              cudaStream_t stream);
+cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
+                                bool pdl, bool gather, cudaStream_t stream);
+
+struct FfnMaps {
+  CUtensorMap w_gu;   // [E*2I rows, H cols] bf16, box 64 x 64
+  CUtensorMap w_down; // [E*H rows, I cols] bf16, box 64 x 64
+  CUtensorMap xp;     // [B*k rows, H cols] bf16, box 64 x 16
+  CUtensorMap act;    // [B*k rows, I cols] bf16, box 64 x 16
+};
+
+cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
+                              __nv_bfloat16 *out, int grid, bool pdl,
+                              cudaStream_t stream);
+
+#if defined(__CUDACC__)
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Programmatic dependent launch.
+__device__ __forceinline__ void pdl_wait_primary() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// mbarrier ------------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar,
+                                                      uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(
+                   bar),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false after `timeout_ns` or once *abort is set.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  volatile int *abort,
+                                                  uint64_t timeout_ns) {
+#pragma unroll 1
+  for (int i = 0; i < 256; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+#pragma unroll 1
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
+}
+
+// Bounded wait that ignores the abort flag (used to drain after an abort).
+__device__ __forceinline__ bool mbar_wait_timeout(uint32_t bar, uint32_t parity,
+                                                  uint64_t timeout_ns) {
+  const uint64_t t0 = global_timer_ns();
+#pragma unroll 1
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
+}
+
+// TMA -----------------------------------------------------------------------
+__device__ __forceinline__ void tma_prefetch_desc(const void *map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+// 2-D tiled load; x = innermost (element) coordinate, y = row.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map,
+                                            uint32_t bar, int x, int y,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_"
+      "tx::bytes.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// tcgen05 -------------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile(
+      "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+          dst_smem),
+      "r"(ncols)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(
+                   taddr),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc,
+                                            uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
+          d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on `bar` once every previously issued MMA of this thread completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 "
+      "[%0];" ::"r"(bar)
+      : "memory");
+}
+// 32 lanes x 32 bit, 16 consecutive columns per thread.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, "
+      "[%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]),
+        "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]),
+        "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]),
+        "=r"(v[15])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle,
+// 8-row core groups 1024 bytes apart (SBO), tile base 1024-byte aligned.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address
+  d |= (uint64_t)1 << 16;                     // LBO (unused for SW128 K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;           // SBO
+  d |= (uint64_t)1 << 46;                     // descriptor version (sm_100 family)
+  d |= (uint64_t)2 << 61;                     // SWIZZLE_128B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major.
+__device__ __forceinline__ uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4)                       // D format: fp32
+         | (1u << 7)                     // A format: bf16
+         | (1u << 10)                    // B format: bf16
+         | ((uint32_t)(N >> 3) << 17)    // N / 8
+         | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+#endif  // __CUDACC__
+
+}  // namespace slimwise

@@ -1,0 +1,483 @@
+// expert_ffn.cu -- grouped SwiGLU expert FFN over the selected-expert union,
+// with the gate-weighted combine fused into its epilogue.
+//
+// Decode reads the weights of every expert in the union of the batch's
+// selections once per step (SlimWise Sec. 2.1, Eq. 1) and each expert sees
+// few tokens (Sec. 2.1: about B*k/m per step), so the kernel is a weight
+// stream: HBM -> (TMA, 128-byte swizzle) -> shared-memory ring ->
+// tcgen05.mma with the weights as the M = 128 operand and the expert's
+// tokens as the N operand (16..256, padded to 16) -> TMEM accumulators ->
+// epilogue warps.
+//
+// One persistent CTA per SM (192 threads):
+//   warp 0   producer: takes work items from a global counter, waits for a
+//            down item's activations, issues the TMA loads of each stage.
+//   warp 1   MMA issuer (one thread) and TMEM owner; double-buffered
+//            accumulators so the epilogue of one item overlaps the next.
+//   warps 2-5 epilogue (128 threads, TMEM lane quarters 2,3,0,1).
+// Work items, all of gate/up before any of down (so a down item only waits
+// for work that has already been handed out):
+//   gate/up (entry, i-tile): A = 64 gate rows + the matching 64 up rows of
+//            W_gu[e], K = H; epilogue computes act = SiLU(gate) * up (fp32),
+//            stores bf16 act in grouped order and counts the tile done.
+//   down    (entry, h-tile): A = 128 rows of W_down[e], K = I, B = act of the
+//            entry's tokens (after all its gate/up tiles are done); epilogue
+//            stores fp32 y; the last of the k contributions to a
+//            (token, h-tile) sums sum_j g[t,j] y_j in j order and writes bf16.
+// Every wait is bounded (1 s): on timeout the CTA records an error bit in the
+// workspace, stops taking work, drains its own copies and MMAs, frees TMEM
+// and exits.
+#include "common.cuh"
+
+namespace slimwise {
+
+constexpr int kFfnThreads = 192;
+constexpr int kEpiThreads = 128;
+constexpr int kItemRing = 4;
+constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
+constexpr int kXchBytes = 2 * kTileRows * kXchStride * 4;
+constexpr uint64_t kTimeoutNs = 1000000000ull;
+
+struct FfnSmem {
+  int stages;
+  int stage_bytes;
+  size_t xch_off, bar_off, misc_off, total;
+};
+
+__host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
+  FfnSmem p;
+  p.stages = stages;
+  p.stage_bytes = kATileBytes + tok_chunk * kBlockK * 2;
+  p.xch_off = (size_t)stages * p.stage_bytes;
+  p.bar_off = p.xch_off + kXchBytes;
+  // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
+  p.misc_off = p.bar_off + 8 * (2 * stages + 4 + 2 * kItemRing + 1);
+  // item ring, tmem base, abort, consumed stages, combine list count + list
+  p.total = p.misc_off + 4 * (kItemRing + 4) + 4 * kMaxTokTile + 1024;
+  return p;
+}
+
+struct Item {
+  int down;      // 0: gate/up, 1: down
+  int entry;
+  int tile;
+  int expert;
+  int slot_base;
+  int n;         // tokens
+  int n16;       // tokens rounded up to 16, / 16
+};
+
+__device__ __forceinline__ Item decode_item(int item, int items1, int t1,
+                                            int t2, const Ws &ws) {
+  Item it;
+  if (item < items1) {
+    it.down = 0;
+    it.entry = item / t1;
+    it.tile = item - it.entry * t1;
+  } else {
+    const int j = item - items1;
+    it.down = 1;
+    it.entry = j / t2;
+    it.tile = j - it.entry * t2;
+  }
+  const int4 en = __ldcg(&ws.entries[it.entry]);
+  it.expert = en.x;
+  it.slot_base = en.y;
+  it.n = en.z;
+  it.n16 = (en.z + 15) >> 4;
+  return it;
+}
+
+__device__ __forceinline__ void epi_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire(const int *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit) {
+  *abort = 1;
+  atomicOr(&ws.ctrl[kCtrlErr], bit);
+}
+
+__global__ void __launch_bounds__(kFfnThreads, 1)
+    expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
+                      __nv_bfloat16 *__restrict__ out, int stages,
+                      int tmem_cols) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char *smem = reinterpret_cast<unsigned char *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const FfnSmem plan = ffn_smem_plan(d.tok_chunk, stages);
+  const uint32_t smem_base = smem_u32(smem);
+  float *xch = reinterpret_cast<float *>(smem + plan.xch_off);
+  const uint32_t bar0 = smem_base + (uint32_t)plan.bar_off;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (stages + s); };
+  auto accf_bar = [&](int b) { return bar0 + 8u * (2 * stages + b); };
+  auto acce_bar = [&](int b) { return bar0 + 8u * (2 * stages + 2 + b); };
+  auto itf_bar = [&](int r) { return bar0 + 8u * (2 * stages + 4 + r); };
+  auto ite_bar = [&](int r) { return bar0 + 8u * (2 * stages + 4 + kItemRing + r); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * stages + 4 + 2 * kItemRing);
+  int *misc = reinterpret_cast<int *>(smem + plan.misc_off);
+  volatile int *ring = misc;                         // [kItemRing]
+  volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc + kItemRing);
+  volatile int *abort = misc + kItemRing + 1;
+  volatile int *consumed = misc + kItemRing + 2;     // stages the MMA finished with
+  int *comb_n = misc + kItemRing + 3;
+  int *comb_list = misc + kItemRing + 4;             // [kMaxTokTile]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accf_bar(b), 1);
+      mbar_init(acce_bar(b), kEpiThreads);
+    }
+    for (int r = 0; r < kItemRing; ++r) {
+      mbar_init(itf_bar(r), 1);
+      mbar_init(ite_bar(r), 1 + kEpiThreads);
+    }
+    mbar_init(drain_bar, 1);
+    *abort = 0;
+    *consumed = 0;
+    *comb_n = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&maps.w_gu);
+    tma_prefetch_desc(&maps.w_down);
+    tma_prefetch_desc(&maps.xp);
+    tma_prefetch_desc(&maps.act);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32((const void *)tmem_slot), (uint32_t)tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  // Everything below reads the grouping kernel's results.
+  pdl_wait_primary();
+
+  const int items1 = __ldcg(&ws.ctrl[kCtrlItems1]);
+  const int total = __ldcg(&ws.ctrl[kCtrlTotalItems]);
+  const int t1 = d.I / kGateRows;
+  const int t2 = d.H / kTileRows;
+  const int nb_cols = d.tok_chunk;  // TMEM columns per accumulator buffer
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_x = l2_policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      int slot = 0;
+      uint32_t rphase = 0;
+      int issued = 0;
+      for (;;) {
+        int item = atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
+        if (*abort) item = 0x7FFFFFFF;
+        if (!mbar_wait_bounded(ite_bar(slot), rphase ^ 1u, abort, kTimeoutNs)) {
+          if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+          break;
+        }
+        ring[slot] = item;
+        mbar_arrive(itf_bar(slot));
+        if (++slot == kItemRing) {
+          slot = 0;
+          rphase ^= 1u;
+        }
+        if (item >= total) break;
+        const Item it = decode_item(item, items1, t1, t2, ws);
+        if (it.down) {
+          // the entry's activations must be complete: all its gate/up tiles
+          const int *done = &ws.entry_done[it.entry];
+          bool ok = ld_acquire(done) >= t1;
+          if (!ok) {
+            const uint64_t t0 = global_timer_ns();
+            while (!(ok = ld_acquire(done) >= t1)) {
+              if (*abort) break;
+              if (global_timer_ns() - t0 > kTimeoutNs) {
+                raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
+                break;
+              }
+              __nanosleep(128);
+            }
+          }
+          if (!ok) break;
+          fence_proxy_async_global();
+        }
+        const int nk = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const void *amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
+        const void *bmap = it.down ? (const void *)&maps.act : (const void *)&maps.xp;
+        int row0, row1;
+        if (it.down) {
+          row0 = it.expert * d.H + it.tile * kTileRows;
+          row1 = row0 + kGateRows;
+        } else {
+          row0 = it.expert * 2 * d.I + it.tile * kGateRows;
+          row1 = row0 + d.I;
+        }
+        const uint32_t bytes = (uint32_t)(kATileBytes + it.n16 * kTokBox * kBlockK * 2);
+        bool ok = true;
+        for (int kc = 0; kc < nk; ++kc) {
+          if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, kTimeoutNs)) {
+            if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+            ok = false;
+            break;
+          }
+          const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
+          const uint32_t b = a + kATileBytes;
+          mbar_arrive_expect_tx(full_bar(stage), bytes);
+          tma_load_2d(a, amap, full_bar(stage), kc * kBlockK, row0, pol_w);
+          tma_load_2d(a + kATileBytes / 2, amap, full_bar(stage), kc * kBlockK, row1, pol_w);
+          for (int j = 0; j < it.n16; ++j)
+            tma_load_2d(b + j * (kTokBox * kBlockK * 2), bmap, full_bar(stage),
+                        kc * kBlockK, it.slot_base + j * kTokBox, pol_x);
+          ++issued;
+          if (++stage == stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+      }
+      if (*abort) {
+        // let this CTA's copies in flight land before shared memory goes away
+        for (int s = *consumed; s < issued; ++s)
+          mbar_wait_timeout(full_bar(s % stages), (uint32_t)((s / stages) & 1), 10000000ull);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int slot = 0;
+      uint32_t rphase = 0;
+      int n_consumed = 0;
+      bool issued_any = false;
+      for (int local = 0;; ++local) {
+        if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, kTimeoutNs)) {
+          if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+          break;
+        }
+        const int item = ring[slot];
+        mbar_arrive(ite_bar(slot));
+        if (++slot == kItemRing) {
+          slot = 0;
+          rphase ^= 1u;
+        }
+        if (item >= total) break;
+        const Item it = decode_item(item, items1, t1, t2, ws);
+        const int b = local & 1;
+        const uint32_t use = (uint32_t)(local >> 1);
+        if (!mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, kTimeoutNs)) {
+          if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(b * nb_cols);
+        const uint32_t idesc = idesc_bf16_f32(kTileRows, it.n16 * kTokBox);
+        const int nk = it.down ? d.I / kBlockK : d.H / kBlockK;
+        bool ok = true;
+        for (int kc = 0; kc < nk; ++kc) {
+          if (!mbar_wait_bounded(full_bar(stage), phase, abort, kTimeoutNs)) {
+            if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
+          const uint32_t bb = a + kATileBytes;
+#pragma unroll
+          for (int kk = 0; kk < kBlockK / 16; ++kk)
+            tc_mma_bf16(d_tmem, smem_desc_sw128(a + kk * 32),
+                        smem_desc_sw128(bb + kk * 32), idesc,
+                        (kc | kk) != 0 ? 1u : 0u);
+          tc_commit(empty_bar(stage));
+          issued_any = true;
+          *consumed = ++n_consumed;
+          if (++stage == stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        tc_commit(accf_bar(b));
+      }
+      if (*abort && issued_any) {
+        tc_commit(drain_bar);
+        mbar_wait_timeout(drain_bar, 0, 10000000ull);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;             // TMEM lane quarter of this warp
+    const int row = 32 * q + lane;      // accumulator row = TMEM lane
+    const int et = threadIdx.x - 64;    // 0..127
+    int slot = 0;
+    uint32_t rphase = 0;
+    for (int local = 0;; ++local) {
+      if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, kTimeoutNs)) {
+        if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+        break;
+      }
+      const int item = ring[slot];
+      mbar_arrive(ite_bar(slot));
+      if (++slot == kItemRing) {
+        slot = 0;
+        rphase ^= 1u;
+      }
+      if (item >= total) break;
+      const Item it = decode_item(item, items1, t1, t2, ws);
+      const int b = local & 1;
+      const uint32_t use = (uint32_t)(local >> 1);
+      if (!mbar_wait_bounded(accf_bar(b), use & 1u, abort, kTimeoutNs)) {
+        if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * nb_cols);
+      if (!it.down) {
+        // gate rows live in TMEM lanes 0..63, the matching up rows in 64..127
+        const int n_loc = et >> 3;          // token column within a 16-chunk
+        const int i0 = (et & 7) * 8;        // 8 consecutive intermediate indices
+        for (int c = 0; c < it.n16; ++c) {
+          uint32_t v[16];
+          tmem_ld16(taddr + c * 16, v);
+          tmem_ld_wait();
+          float *xb = xch + (c & 1) * kTileRows * kXchStride;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) xb[row * kXchStride + j] = __uint_as_float(v[j]);
+          epi_bar();
+          const int col = c * 16 + n_loc;
+          if (col < it.n) {
+            uint32_t packed[4];
+#pragma unroll
+            for (int ii = 0; ii < 8; ii += 2) {
+              float a2[2];
+#pragma unroll
+              for (int u2 = 0; u2 < 2; ++u2) {
+                const float g = xb[(i0 + ii + u2) * kXchStride + n_loc];
+                const float u = xb[(kGateRows + i0 + ii + u2) * kXchStride + n_loc];
+                a2[u2] = g / (1.0f + expf(-g)) * u;
+              }
+              __nv_bfloat162 h2 = __floats2bfloat162_rn(a2[0], a2[1]);
+              packed[ii / 2] = *reinterpret_cast<uint32_t *>(&h2);
+            }
+            *reinterpret_cast<uint4 *>(ws.act + (size_t)(it.slot_base + col) * d.I +
+                                       it.tile * kGateRows + i0) =
+                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(acce_bar(b));
+        // publish the activations to the TMA (async proxy) readers of any CTA
+        fence_proxy_async_global();
+        __threadfence();
+        epi_bar();
+        if (et == 0) atomicAdd(&ws.entry_done[it.entry], 1);
+      } else {
+        const int h = it.tile * kTileRows + row;
+        for (int c = 0; c < it.n16; ++c) {
+          uint32_t v[16];
+          tmem_ld16(taddr + c * 16, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int col = c * 16 + j;
+            if (col < it.n)
+              ws.y[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(acce_bar(b));
+        __threadfence();
+        if (et == 0) *comb_n = 0;
+        epi_bar();
+        // count this contribution for each token; the k-th one combines
+        for (int col = et; col < it.n; col += kEpiThreads) {
+          const int s = __ldcg(&ws.perm[it.slot_base + col]);
+          const int t = s / d.k;
+          const int old = atomicAdd(&ws.comb_cnt[(size_t)t * t2 + it.tile], 1);
+          if (old == d.k - 1) comb_list[atomicAdd(comb_n, 1)] = t;
+        }
+        __threadfence();
+        epi_bar();
+        const int n_list = *comb_n;
+        const int hh = it.tile * kCombineTile + et;
+        for (int i = 0; i < n_list; ++i) {
+          const int t = comb_list[i];
+          float acc = 0.0f;
+          for (int j = 0; j < d.k; ++j) {
+            const int p = __ldcg(&ws.pos[(size_t)t * d.k + j]);
+            const float g = __ldcg(&ws.topk_gate[(size_t)t * d.k + j]);
+            acc = fmaf(g, __ldcg(&ws.y[(size_t)p * d.H + hh]), acc);
+          }
+          out[(size_t)t * d.H + hh] = __float2bfloat16_rn(acc);
+        }
+        epi_bar();
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, (uint32_t)tmem_cols);
+  }
+}
+
+int ffn_stages_for(int tok_chunk, size_t smem_limit) {
+  int s = 8;
+  while (s > 2 && ffn_smem_plan(tok_chunk, s).total + 1024 > smem_limit) --s;
+  return s;
+}
+
+cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
+                              __nv_bfloat16 *out, int grid, bool pdl,
+                              cudaStream_t stream) {
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  int optin = 0;
+  err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (err != cudaSuccess) return err;
+  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin);
+  const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
+  if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
+  err = cudaFuncSetAttribute(expert_ffn_kernel,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  int tmem_cols = 32;
+  while (tmem_cols < 2 * d.tok_chunk) tmem_cols <<= 1;
+
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kFfnThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, expert_ffn_kernel, maps, d, ws, out, stages,
+                            tmem_cols);
+}
+
+}  // namespace slimwise

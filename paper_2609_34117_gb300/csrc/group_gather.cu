@@ -1,0 +1,176 @@
+// group_gather.cu -- grouping of the B*k routed (token, slot) pairs by expert
+// and gather of the hidden rows into that grouped order.
+//
+// A decode step must read the weights of the union of experts selected
+// across the batch (SlimWise Sec. 2.1, Eq. 1).  This kernel turns the top-k
+// selections into:
+//   counts[e]  histogram of selections,
+//   offsets    exclusive scan of counts (expert ascending),
+//   union_ids  selected experts ascending, union size U,
+//   perm/pos   grouped order of the slots: (expert asc, token asc),
+//   entries    the FFN kernel's work list: one entry per (expert, chunk of
+//              at most tok_chunk tokens),
+//   xp         hidden rows copied into grouped order, so the FFN kernel can
+//              stream each expert's tokens with plain 2-D TMA boxes.
+// Every CTA recomputes the histogram of the whole batch (B*k ids, a few KB
+// from L2) so the rank of a slot inside its expert, its token-order prefix
+// count, is known without a grid-wide barrier; integer counts make the
+// result independent of atomic arrival order.
+#include "common.cuh"
+
+namespace slimwise {
+
+constexpr int kGroupTokens = 4;
+constexpr int kGroupThreads = 512;
+
+// Exclusive scan of vals[0..n) (n <= kMaxExperts) into outp[0..n], by one
+// warp; returns the total.  Each lane scans a contiguous run.
+__device__ int warp_exclusive_scan(const int *vals, int *outp, int n, int lane) {
+  const int per = (n + 31) / 32;
+  const int lo = min(n, lane * per), hi = min(n, lo + per);
+  int local = 0;
+  for (int i = lo; i < hi; ++i) local += vals[i];
+  int incl = local;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    int o = __shfl_up_sync(0xFFFFFFFFu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  int run = incl - local;
+  for (int i = lo; i < hi; ++i) {
+    outp[i] = run;
+    run += vals[i];
+  }
+  const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  if (lane == 0) outp[n] = total;
+  return total;
+}
+
+__global__ void __launch_bounds__(kGroupThreads)
+    group_gather_kernel(const __nv_bfloat16 *__restrict__ hidden, Dims d, Ws ws,
+                        int do_gather) {
+  __shared__ int cnt_all[kMaxExperts];
+  __shared__ int cnt_before[kMaxExperts];
+  __shared__ int offs[kMaxExperts + 1];
+  __shared__ int flag_scan[kMaxExperts + 1];
+  __shared__ int chunk_cnt[kMaxExperts];
+  __shared__ int entry_base[kMaxExperts + 1];
+  __shared__ int my_pos[kGroupTokens * kMaxTopK];
+  __shared__ int bad;
+
+  // Wait for the routing kernel's results; then let the FFN kernel's CTAs
+  // start their prologue.
+  pdl_wait_primary();
+  pdl_launch_dependents();
+
+  const int B = d.B, k = d.k, E = d.E, H = d.H;
+  const int S = B * k;
+  const int t0 = blockIdx.x * kGroupTokens;
+  const int t1 = min(B, t0 + kGroupTokens);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  for (int e = tid; e < E; e += blockDim.x) {
+    cnt_all[e] = 0;
+    cnt_before[e] = 0;
+  }
+  if (tid == 0) bad = 0;
+  __syncthreads();
+  for (int s = tid; s < S; s += blockDim.x) {
+    int e = ws.topk_idx[s];
+    if (e < 0 || e >= E) {  // only possible for caller-given selections
+      bad = SLIMWISE_DEVERR_BAD_TOPK;
+      e = min(max(e, 0), E - 1);
+    }
+    atomicAdd(&cnt_all[e], 1);
+    if (s < t0 * k) atomicAdd(&cnt_before[e], 1);
+  }
+  __syncthreads();
+  if (warp == 0) warp_exclusive_scan(cnt_all, offs, E, lane);
+  __syncthreads();
+
+  // Grouped position of each of this CTA's slots: offset of the expert plus
+  // the number of earlier tokens that selected it.
+  if (tid == 0) {
+    for (int t = t0; t < t1; ++t)
+      for (int j = 0; j < k; ++j) {
+        int e = min(max(ws.topk_idx[t * k + j], 0), E - 1);
+        my_pos[(t - t0) * k + j] = offs[e] + cnt_before[e]++;
+      }
+  }
+  __syncthreads();
+  const int nslots = (t1 - t0) * k;
+  for (int i = tid; i < nslots; i += blockDim.x) {
+    const int s = t0 * k + i, p = my_pos[i];
+    ws.pos[s] = p;
+    ws.perm[p] = s;
+  }
+  if (do_gather) {
+    const int vecs = H / 8;  // 16-byte vectors per row
+    for (int i = tid; i < nslots * vecs; i += blockDim.x) {
+      const int r = i / vecs, v = i - r * vecs;
+      const int t = t0 + r / k;
+      reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[r] * H)[v] =
+          reinterpret_cast<const uint4 *>(hidden + (size_t)t * H)[v];
+    }
+  }
+  const int ht = H / kCombineTile;
+  for (int i = tid; i < (t1 - t0) * ht; i += blockDim.x)
+    ws.comb_cnt[(size_t)t0 * ht + i] = 0;
+
+  if (blockIdx.x != 0) return;
+
+  // CTA 0 publishes the batch-wide results and the FFN work list.
+  for (int e = tid; e < E; e += blockDim.x) {
+    ws.counts[e] = cnt_all[e];
+    ws.offsets[e] = offs[e];
+    cnt_before[e] = cnt_all[e] > 0 ? 1 : 0;  // reuse as union flags
+    chunk_cnt[e] = (cnt_all[e] + d.tok_chunk - 1) / d.tok_chunk;
+  }
+  if (tid == 0) ws.offsets[E] = offs[E];
+  __syncthreads();
+  if (warp == 0) warp_exclusive_scan(cnt_before, flag_scan, E, lane);
+  if (warp == 1) warp_exclusive_scan(chunk_cnt, entry_base, E, lane);
+  __syncthreads();
+  const int U = flag_scan[E];
+  const int n_entries = entry_base[E];
+  for (int e = tid; e < E; e += blockDim.x) {
+    if (cnt_before[e]) ws.union_ids[flag_scan[e]] = e;
+    if (e >= U) ws.union_ids[e] = -1;
+    const int n_e = offs[e + 1] - offs[e];
+    for (int c = 0; c < chunk_cnt[e]; ++c) {
+      const int base = c * d.tok_chunk;
+      ws.entries[entry_base[e] + c] =
+          make_int4(e, offs[e] + base, min(d.tok_chunk, n_e - base), 0);
+    }
+  }
+  for (int i = tid; i < n_entries; i += blockDim.x) ws.entry_done[i] = 0;
+  if (tid == 0) {
+    const int t1_items = d.I / kGateRows;
+    const int t2_items = d.H / kTileRows;
+    ws.ctrl[kCtrlUnionSize] = U;
+    ws.ctrl[kCtrlNumEntries] = n_entries;
+    ws.ctrl[kCtrlItems1] = n_entries * t1_items;
+    ws.ctrl[kCtrlTotalItems] = n_entries * (t1_items + t2_items);
+    ws.ctrl[kCtrlWorkCounter] = 0;
+  }
+  __syncthreads();
+  if (tid == 0 && bad) atomicOr(&ws.ctrl[kCtrlErr], bad);
+}
+
+cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
+                                bool pdl, bool gather, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((d.B + kGroupTokens - 1) / kGroupTokens);
+  cfg.blockDim = dim3(kGroupThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, group_gather_kernel, hidden, d, ws,
+                            gather ? 1 : 0);
+}
+
+}  // namespace slimwise

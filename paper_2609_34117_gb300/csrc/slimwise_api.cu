@@ -1,0 +1,306 @@
+// slimwise_api.cu -- the C ABI declared in include/slimwise_moe.h: argument
+// checks, workspace layout, TMA descriptors, and the three launches of one
+// decode MoE layer (route/top-k -> group/gather -> expert FFN + combine).
+#include <mutex>
+
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+
+using namespace slimwise;
+
+namespace {
+
+struct DeviceInfo {
+  int sms = 0;
+  int smem_optin = 0;
+  bool ready = false;
+};
+
+std::mutex g_mu;
+DeviceInfo g_dev[64];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int device_info(DeviceInfo *out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+    return SLIMWISE_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mu);
+  DeviceInfo &di = g_dev[dev];
+  if (!di.ready) {
+    if (cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&di.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess)
+      return SLIMWISE_ERR_CUDA;
+    di.ready = true;
+  }
+  if (!g_encode) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                         cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return SLIMWISE_ERR_CUDA;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  *out = di;
+  return SLIMWISE_OK;
+}
+
+// 2-D bf16 tensor map: `rows` x `cols` row-major, box `box_rows` x 64,
+// 128-byte swizzle, zero fill outside the tensor.
+int encode_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
+               uint32_t box_rows) {
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kBlockK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? SLIMWISE_OK : SLIMWISE_ERR_CUDA;
+}
+
+bool aligned(const void *p, uintptr_t a) {
+  return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0;
+}
+
+int check_shape(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
+  if (!s) return SLIMWISE_ERR_INVALID_ARG;
+  if (s->num_tokens < 0 || s->num_tokens > (1 << 20)) return SLIMWISE_ERR_INVALID_ARG;
+  if (s->hidden < 128 || s->hidden % 128 != 0 || s->hidden > 65536)
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  if (s->inter < 64 || s->inter % 64 != 0 || s->inter > 65536)
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  if (s->num_experts < 1 || s->num_experts > kMaxExperts)
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  if (m_ret < 1 || m_ret > s->num_experts) return SLIMWISE_ERR_INVALID_ARG;
+  if (top_k < 1 || top_k > kMaxTopK || top_k > m_ret) return SLIMWISE_ERR_INVALID_ARG;
+  if ((uint64_t)s->num_experts * 2 * s->inter > 0xFFFFFFFFull ||
+      (uint64_t)s->num_experts * s->hidden > 0xFFFFFFFFull)
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  return SLIMWISE_OK;
+}
+
+Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
+  Dims d;
+  d.B = s->num_tokens;
+  d.H = s->hidden;
+  d.E = s->num_experts;
+  d.I = s->inter;
+  d.k = top_k;
+  d.m_ret = m_ret;
+  d.tok_chunk = token_chunk_for(d.B);
+  return d;
+}
+
+int check_workspace(const slimwise_moe_shape *s, int32_t top_k, void *ws,
+                    size_t ws_bytes, WsLayout *L) {
+  if (!ws) return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(ws, 256)) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  *L = make_layout(s->num_tokens, s->hidden, s->num_experts, s->inter, top_k);
+  return ws_bytes >= L->total ? SLIMWISE_OK : SLIMWISE_ERR_WORKSPACE;
+}
+
+int copy_out(void *dst, const void *src, size_t bytes, cudaStream_t st) {
+  if (!dst || !bytes) return SLIMWISE_OK;
+  return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, st) == cudaSuccess
+             ? SLIMWISE_OK
+             : SLIMWISE_ERR_CUDA;
+}
+
+int copy_group_outputs(const Ws &w, const Dims &d, cudaStream_t st, int32_t *counts,
+                       int32_t *offsets, int32_t *union_ids, int32_t *union_size,
+                       int32_t *perm, int32_t *pos) {
+  const size_t slots = (size_t)d.B * d.k;
+  int rc = SLIMWISE_OK;
+  if (!rc) rc = copy_out(counts, w.counts, (size_t)d.E * 4, st);
+  if (!rc) rc = copy_out(offsets, w.offsets, (size_t)(d.E + 1) * 4, st);
+  if (!rc) rc = copy_out(union_ids, w.union_ids, (size_t)d.E * 4, st);
+  if (!rc) rc = copy_out(union_size, w.ctrl + kCtrlUnionSize, 4, st);
+  if (!rc) rc = copy_out(perm, w.perm, slots * 4, st);
+  if (!rc) rc = copy_out(pos, w.pos, slots * 4, st);
+  return rc;
+}
+
+int decode_impl(const void *hidden, const float *router_w, const int32_t *retained,
+                int32_t n_retained, const void *w_gate_up, const void *w_down,
+                int32_t top_k, void *out, void *stream, const slimwise_moe_shape *shape,
+                void *workspace, size_t workspace_bytes, const slimwise_decode_opts *opts) {
+  const int32_t m_ret = retained ? n_retained : (shape ? shape->num_experts : 0);
+  int rc = check_shape(shape, top_k, m_ret);
+  if (rc) return rc;
+  if (shape->num_tokens == 0) return SLIMWISE_OK;
+  if (!hidden || !router_w || !w_gate_up || !w_down || !out) return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(router_w, 16) || !aligned(w_gate_up, 16) ||
+      !aligned(w_down, 16) || !aligned(out, 16) || (retained && !aligned(retained, 4)))
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  WsLayout L;
+  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L);
+  if (rc) return rc;
+  DeviceInfo di;
+  rc = device_info(&di);
+  if (rc) return rc;
+
+  const Dims d = make_dims(shape, top_k, m_ret);
+  const Ws w = make_ws(workspace, L);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const bool pdl = !(opts && opts->disable_pdl);
+  int grid = di.sms;
+  if (opts && opts->grid_ctas > 0) grid = opts->grid_ctas;
+
+  FfnMaps maps;
+  const uint64_t slots = (uint64_t)d.B * d.k;
+  if (encode_map(&maps.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
+      encode_map(&maps.w_down, w_down, (uint64_t)d.E * d.H, d.I, kGateRows) ||
+      encode_map(&maps.xp, w.xp, slots, d.H, kTokBox) ||
+      encode_map(&maps.act, w.act, slots, d.I, kTokBox))
+    return SLIMWISE_ERR_CUDA;
+
+  if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained,
+                        d, w, st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  if (launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), d, w, pdl, true,
+                          st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  const bool timed = opts && opts->ffn_begin && opts->ffn_end;
+  if (timed && cudaEventRecord(static_cast<cudaEvent_t>(opts->ffn_begin), st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  if (launch_expert_ffn(maps, d, w, static_cast<__nv_bfloat16 *>(out), grid,
+                        pdl && !timed, st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  if (timed && cudaEventRecord(static_cast<cudaEvent_t>(opts->ffn_end), st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  return SLIMWISE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *slimwise_status_string(int status) {
+  switch (status) {
+    case SLIMWISE_OK: return "ok";
+    case SLIMWISE_ERR_INVALID_ARG: return "invalid argument";
+    case SLIMWISE_ERR_UNSUPPORTED_SHAPE: return "unsupported shape or alignment";
+    case SLIMWISE_ERR_WORKSPACE: return "workspace too small";
+    case SLIMWISE_ERR_CUDA: return "CUDA error";
+    case SLIMWISE_ERR_DEVICE: return "device-side error";
+    default: return "unknown status";
+  }
+}
+
+int slimwise_moe_workspace_size(const slimwise_moe_shape *shape, int32_t top_k,
+                                size_t *bytes) {
+  if (!bytes) return SLIMWISE_ERR_INVALID_ARG;
+  int rc = check_shape(shape, top_k, shape ? shape->num_experts : 0);
+  if (rc) return rc;
+  *bytes = make_layout(shape->num_tokens, shape->hidden, shape->num_experts,
+                       shape->inter, top_k)
+               .total;
+  return SLIMWISE_OK;
+}
+
+int slimwise_moe_decode(const void *hidden, const float *router_w,
+                        const int32_t *retained_idx, int32_t n_retained,
+                        const void *w_gate_up, const void *w_down, int32_t top_k,
+                        void *out, void *stream, const slimwise_moe_shape *shape,
+                        void *workspace, size_t workspace_bytes) {
+  if (!retained_idx) return SLIMWISE_ERR_INVALID_ARG;
+  return decode_impl(hidden, router_w, retained_idx, n_retained, w_gate_up, w_down,
+                     top_k, out, stream, shape, workspace, workspace_bytes, nullptr);
+}
+
+int slimwise_moe_decode_full(const void *hidden, const float *router_w,
+                             const void *w_gate_up, const void *w_down, int32_t top_k,
+                             void *out, void *stream, const slimwise_moe_shape *shape,
+                             void *workspace, size_t workspace_bytes) {
+  return decode_impl(hidden, router_w, nullptr, 0, w_gate_up, w_down, top_k, out, stream,
+                     shape, workspace, workspace_bytes, nullptr);
+}
+
+int slimwise_moe_decode_ex(const void *hidden, const float *router_w,
+                           const int32_t *retained_idx, int32_t n_retained,
+                           const void *w_gate_up, const void *w_down, int32_t top_k,
+                           void *out, void *stream, const slimwise_moe_shape *shape,
+                           void *workspace, size_t workspace_bytes,
+                           const slimwise_decode_opts *opts) {
+  return decode_impl(hidden, router_w, retained_idx, n_retained, w_gate_up, w_down, top_k,
+                     out, stream, shape, workspace, workspace_bytes, opts);
+}
+
+int slimwise_moe_route(const void *hidden, const float *router_w,
+                       const int32_t *retained_idx, int32_t n_retained, int32_t top_k,
+                       void *stream, const slimwise_moe_shape *shape, void *workspace,
+                       size_t workspace_bytes, int32_t *topk_idx, float *topk_gate,
+                       int32_t *counts, int32_t *offsets, int32_t *union_ids,
+                       int32_t *union_size, int32_t *perm, int32_t *pos) {
+  const int32_t m_ret = retained_idx ? n_retained : (shape ? shape->num_experts : 0);
+  int rc = check_shape(shape, top_k, m_ret);
+  if (rc) return rc;
+  if (shape->num_tokens == 0) return SLIMWISE_OK;
+  if (!hidden || !router_w) return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(router_w, 16)) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  WsLayout L;
+  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L);
+  if (rc) return rc;
+  DeviceInfo di;
+  rc = device_info(&di);
+  if (rc) return rc;
+  const Dims d = make_dims(shape, top_k, m_ret);
+  const Ws w = make_ws(workspace, L);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained_idx,
+                        d, w, st) != cudaSuccess ||
+      launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), d, w, false, false,
+                          st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  const size_t slots = (size_t)d.B * d.k;
+  rc = copy_out(topk_idx, w.topk_idx, slots * 4, st);
+  if (!rc) rc = copy_out(topk_gate, w.topk_gate, slots * 4, st);
+  if (!rc) rc = copy_group_outputs(w, d, st, counts, offsets, union_ids, union_size, perm, pos);
+  return rc;
+}
+
+int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
+                       const slimwise_moe_shape *shape, void *workspace,
+                       size_t workspace_bytes, int32_t *counts, int32_t *offsets,
+                       int32_t *union_ids, int32_t *union_size, int32_t *perm,
+                       int32_t *pos) {
+  int rc = check_shape(shape, top_k, shape ? shape->num_experts : 0);
+  if (rc) return rc;
+  if (shape->num_tokens == 0) return SLIMWISE_OK;
+  if (!topk_idx) return SLIMWISE_ERR_INVALID_ARG;
+  WsLayout L;
+  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L);
+  if (rc) return rc;
+  DeviceInfo di;
+  rc = device_info(&di);
+  if (rc) return rc;
+  const Dims d = make_dims(shape, top_k, shape->num_experts);
+  const Ws w = make_ws(workspace, L);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const size_t slots = (size_t)d.B * d.k;
+  if (cudaMemsetAsync(w.ctrl + kCtrlErr, 0, 4, st) != cudaSuccess ||
+      cudaMemcpyAsync(w.topk_idx, topk_idx, slots * 4, cudaMemcpyDeviceToDevice, st) !=
+          cudaSuccess ||
+      launch_group_gather(nullptr, d, w, false, false, st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  return copy_group_outputs(w, d, st, counts, offsets, union_ids, union_size, perm, pos);
+}
+
+int slimwise_moe_device_status(const void *workspace, void *stream, int32_t *flags) {
+  if (!workspace || !flags) return SLIMWISE_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  const int32_t *src = static_cast<const int32_t *>(workspace) + kCtrlErr;  // ctrl is first
+  if (cudaMemcpyAsync(&v, src, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  *flags = v;
+  return v ? SLIMWISE_ERR_DEVICE : SLIMWISE_OK;
+}
+
+}  // extern "C"

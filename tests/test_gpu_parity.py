@@ -1,0 +1,289 @@
+"""Parity of the CUDA decode MoE layer (through the C ABI) with the CPU oracle.
+
+Integer results -- top-k ids, union, counts, offsets, grouped permutation --
+must match bit for bit.  Outputs (bf16 in, fp32 accumulate, bf16 out) must be
+within relative L2 error 1e-2 and max-abs error 3e-2 of the oracle's fp64
+values; gates within fp32 rounding of the oracle's.  At the Qwen-class sizes
+the routing of every token is checked and outputs on a seeded sample of
+tokens the oracle evaluates one by one.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_34117_gb300 as sw
+from paper_2609_34117_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+REL_L2_TOL = 1e-2
+MAX_ABS_TOL = 3e-2
+GATE_RTOL = 4e-6
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    sw.build.build()
+    oracle.build()
+
+
+class Layer:
+    def __init__(self, shape, seed=0):
+        self.shape = shape
+        self.w_gu, self.w_d = synth.expert_weights(shape, seed)
+        self.wr = synth.router_weight(shape, seed)
+        self.gu_bits = synth.bf16_bits(self.w_gu)
+        self.d_bits = synth.bf16_bits(self.w_d)
+        self.d_w_gu = self.w_gu.to(DEV)
+        self.d_w_d = self.w_d.to(DEV)
+        self.d_wr = self.wr.to(DEV)
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    return Layer(synth.TINY, seed=0)
+
+
+@pytest.fixture(scope="module")
+def qwen():
+    return Layer(synth.QWEN, seed=0)
+
+
+def _run(layer, x, retained, k, wr=None, workspace=None):
+    wr_d = layer.d_wr if wr is None else wr.to(DEV)
+    xd = x.to(DEV)
+    if retained is None:
+        out = sw.slimwise_moe_decode_full(xd, wr_d, layer.d_w_gu, layer.d_w_d, k, workspace=workspace)
+    else:
+        out = sw.slimwise_moe_decode(xd, wr_d, retained.to(DEV), layer.d_w_gu, layer.d_w_d, k,
+                                     workspace=workspace)
+    route = sw.slimwise_moe_route(xd, wr_d, None if retained is None else retained.to(DEV), k,
+                                  layer.shape.num_experts, layer.shape.inter)
+    torch.cuda.synchronize()
+    return out, {n: t.cpu().numpy() for n, t in route.items()}
+
+
+def _oracle(layer, x, retained, k, tokens=None, wr=None):
+    wr_np = (layer.wr if wr is None else wr).numpy()
+    ret = None if retained is None else retained.numpy()
+    xb = synth.bf16_bits(x)
+    if tokens is None:
+        r = oracle.moe_decode(xb, wr_np, ret, layer.gu_bits, layer.d_bits, k)
+    else:
+        r = oracle.moe_decode_sampled(xb, wr_np, ret, layer.gu_bits, layer.d_bits, k, tokens)
+    r["group"] = oracle.group_by_expert(r["idx"], layer.shape.num_experts)
+    return r
+
+
+def _check_route(route, ref, E):
+    assert np.array_equal(route["topk_idx"], ref["idx"])
+    np.testing.assert_allclose(route["topk_gate"], ref["gates"], rtol=GATE_RTOL, atol=1e-7)
+    g = ref["group"]
+    assert np.array_equal(route["counts"], g["counts"])
+    assert np.array_equal(route["offsets"], g["offsets"])
+    assert int(route["union_size"][0]) == g["union_size"]
+    U = g["union_size"]
+    assert np.array_equal(route["union_ids"][:U], g["union_ids"])
+    assert np.all(route["union_ids"][U:] == -1)
+    assert np.array_equal(route["perm"], g["perm"])
+    assert np.array_equal(route["pos"], g["pos"])
+
+
+def _check_out(got, ref):
+    got = got.astype(np.float64)
+    err = np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30)
+    mx = float(np.abs(got - ref).max()) if ref.size else 0.0
+    assert err <= REL_L2_TOL and mx <= MAX_ABS_TOL, (err, mx)
+    return err, mx
+
+
+def _case(layer, B, m_prime, seed_x, seed_imp, k=None, sample=None, shuffle=False, x=None, wr=None):
+    shape = layer.shape
+    k = shape.top_k if k is None else k
+    if x is None:
+        x = synth.hidden_states(B, shape, seed_x)
+    retained = None if m_prime is None else synth.retained_set(shape.num_experts, m_prime, seed_imp,
+                                                                shuffle=shuffle)
+    out, route = _run(layer, x, retained, k, wr=wr)
+    tokens = None
+    if sample is not None and B > sample:
+        tokens = np.sort(np.random.default_rng(seed_x).choice(B, size=sample, replace=False)).astype(np.int32)
+    ref = _oracle(layer, x, retained, k, tokens=tokens, wr=wr)
+    _check_route(route, ref, shape.num_experts)
+    got = out.float().cpu().numpy()
+    if tokens is not None:
+        got = got[tokens]
+    return _check_out(got, ref["out"]), out, route
+
+
+# --------------------------------------------------------------------------
+def test_tiny_layer_matches_oracle(tiny):
+    (err, mx), _, _ = _case(tiny, B=4, m_prime=8, seed_x=1, seed_imp=2)
+    assert err < 5e-3
+
+
+def test_closed_form_golden_layer():
+    from tests.golden.closed_form import B, E, H, I, build_case
+    case = build_case()
+    with open(os.path.join(os.path.dirname(__file__), "golden", "closed_form_layer.json")) as f:
+        gold = json.load(f)
+    t = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).view(dt).to(DEV)  # noqa: E731
+    x = t(case["x"].view(np.int16), torch.bfloat16)
+    gu = t(case["w_gate_up"].view(np.int16), torch.bfloat16).view(E, 2 * I, H)
+    dn = t(case["w_down"].view(np.int16), torch.bfloat16).view(E, H, I)
+    wr = torch.from_numpy(case["router_w"]).to(DEV)
+    ret = torch.from_numpy(case["retained"]).to(DEV)
+    out = sw.slimwise_moe_decode(x.view(B, H), wr, ret, gu, dn, case["k"])
+    route = sw.slimwise_moe_route(x.view(B, H), wr, ret, case["k"], E, I)
+    torch.cuda.synchronize()
+    assert route["topk_idx"].cpu().tolist() == gold["idx"]
+    np.testing.assert_allclose(route["topk_gate"].cpu().numpy(), np.array(gold["gates"]), rtol=GATE_RTOL)
+    _check_out(out.float().cpu().numpy(), np.array(gold["out"]))
+
+
+def test_qwen_full_pool_b64(qwen):
+    _case(qwen, B=64, m_prime=None, seed_x=1, seed_imp=2, sample=8)
+
+
+@pytest.mark.parametrize("B", [64, 128, 256])
+def test_qwen_pruned_50pct(qwen, B):
+    _case(qwen, B=B, m_prime=64, seed_x=1, seed_imp=2, sample=8)
+
+
+@pytest.mark.parametrize("B,m_prime", [(1, 128), (8, 96), (32, 32), (128, 96), (512, 32), (512, 128)])
+def test_qwen_sweep_points(qwen, B, m_prime):
+    _case(qwen, B=B, m_prime=m_prime, seed_x=1000 + B, seed_imp=2 + m_prime, sample=6)
+
+
+@pytest.mark.parametrize("B", [1, 5, 17, 33, 300])
+def test_ragged_batches_and_token_chunks(tiny, B):
+    # k = m' = 8: every token selects every retained expert, so each expert
+    # holds B tokens and B = 300 exceeds one 256-token work item
+    _case(tiny, B=B, m_prime=8, seed_x=B, seed_imp=2, k=8)
+
+
+@pytest.mark.parametrize("k", [1, 2, 8])
+def test_top_k_extremes(tiny, k):
+    _case(tiny, B=12, m_prime=8, seed_x=7, seed_imp=3, k=k)
+
+
+def test_zero_tokens_is_noop(tiny):
+    x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
+    out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
+    torch.cuda.synchronize()
+    assert out.shape == (0, tiny.shape.hidden)
+
+
+def test_retained_order_irrelevant_and_full_equals_all(qwen):
+    shape = qwen.shape
+    x = synth.hidden_states(64, shape, 11).to(DEV)
+    r_sorted = synth.retained_set(shape.num_experts, 64, 2).to(DEV)
+    r_shuf = synth.retained_set(shape.num_experts, 64, 2, shuffle=True).to(DEV)
+    a = sw.slimwise_moe_decode(x, qwen.d_wr, r_sorted, qwen.d_w_gu, qwen.d_w_d, 8)
+    b = sw.slimwise_moe_decode(x, qwen.d_wr, r_shuf, qwen.d_w_gu, qwen.d_w_d, 8)
+    full = sw.slimwise_moe_decode_full(x, qwen.d_wr, qwen.d_w_gu, qwen.d_w_d, 8)
+    allr = torch.arange(shape.num_experts, dtype=torch.int32, device=DEV).flip(0).contiguous()
+    c = sw.slimwise_moe_decode(x, qwen.d_wr, allr, qwen.d_w_gu, qwen.d_w_d, 8)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    assert torch.equal(full, c)
+
+
+def test_batch_permutation_and_determinism(qwen):
+    shape = qwen.shape
+    x = synth.hidden_states(96, shape, 12).to(DEV)
+    ret = synth.retained_set(shape.num_experts, 64, 2).to(DEV)
+    a = sw.slimwise_moe_decode(x, qwen.d_wr, ret, qwen.d_w_gu, qwen.d_w_d, 8)
+    a2 = sw.slimwise_moe_decode(x, qwen.d_wr, ret, qwen.d_w_gu, qwen.d_w_d, 8)
+    p = torch.randperm(96, generator=torch.Generator().manual_seed(0)).to(DEV)
+    b = sw.slimwise_moe_decode(x[p].contiguous(), qwen.d_wr, ret, qwen.d_w_gu, qwen.d_w_d, 8)
+    torch.cuda.synchronize()
+    assert torch.equal(a, a2)
+    diff = (a[p].float() - b.float()).abs().max().item()
+    assert diff <= 1e-2 * a.float().abs().max().item()
+
+
+def test_workspace_contents_do_not_matter(tiny):
+    shape = tiny.shape
+    x = synth.hidden_states(9, shape, 4).to(DEV)
+    ret = synth.retained_set(shape.num_experts, 8, 2).to(DEV)
+    ws = sw.alloc_workspace(9, shape.hidden, shape.num_experts, shape.inter, 2, DEV)
+    ws.fill_(0xFF)
+    a = sw.slimwise_moe_decode(x, tiny.d_wr, ret, tiny.d_w_gu, tiny.d_w_d, 2, workspace=ws)
+    ws.fill_(0x00)
+    b = sw.slimwise_moe_decode(x, tiny.d_wr, ret, tiny.d_w_gu, tiny.d_w_d, 2, workspace=ws)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    assert sw.slimwise_moe_device_status(ws) == 0
+
+
+def test_duplicate_retained_id_is_reported(tiny):
+    shape = tiny.shape
+    x = synth.hidden_states(4, shape, 4).to(DEV)
+    ret = torch.tensor([1, 3, 3, 7, 9], dtype=torch.int32, device=DEV)
+    ws = sw.alloc_workspace(4, shape.hidden, shape.num_experts, shape.inter, 2, DEV)
+    sw.slimwise_moe_decode(x, tiny.d_wr, ret, tiny.d_w_gu, tiny.d_w_d, 2, workspace=ws)
+    assert sw.slimwise_moe_device_status(ws) & sw.binding.DEVERR_DUPLICATE_RETAINED
+    ok = torch.tensor([1, 3, 7, 9], dtype=torch.int32, device=DEV)
+    sw.slimwise_moe_decode(x, tiny.d_wr, ok, tiny.d_w_gu, tiny.d_w_d, 2, workspace=ws)
+    assert sw.slimwise_moe_device_status(ws) == 0
+
+
+def test_top1_one_hot_router_is_dense_ffn(tiny):
+    shape = tiny.shape
+    ret = synth.retained_set(shape.num_experts, 8, 2)
+    e_star = int(ret[5])
+    x, wr = synth.apply_popularity_bias(synth.hidden_states(16, shape, 5), tiny.wr, torch.zeros(shape.num_experts))
+    wr[e_star, -1] = 8.0
+    out, route = _run(tiny, x, ret, 1, wr=wr)
+    assert np.all(route["topk_idx"][:, 0] == e_star)
+    assert np.all(route["topk_gate"] == 1.0)
+    x64 = x.double().numpy()
+    gu = tiny.w_gu[e_star].double().numpy()
+    dn = tiny.w_d[e_star].double().numpy()
+    I = shape.inter
+    g, u = x64 @ gu[:I].T, x64 @ gu[I:].T
+    ref = (g / (1 + np.exp(-g)) * u) @ dn.T
+    _check_out(out.float().cpu().numpy(), ref)
+
+
+def test_group_of_uniform_selections_matches_oracle_and_eq1():
+    E, k, m_prime, B, draws = 128, 8, 64, 16, 200
+    rng = np.random.default_rng(9)
+    pool = np.sort(rng.choice(E, size=m_prime, replace=False))
+    us = []
+    for _ in range(draws):
+        sel = np.stack([rng.choice(pool, size=k, replace=False) for _ in range(B)]).astype(np.int32)
+        g = sw.slimwise_moe_group(torch.from_numpy(sel).to(DEV), E, hidden=2048, inter=768)
+        ref = oracle.group_by_expert(sel, E)
+        U = int(g["union_size"].item())
+        assert U == ref["union_size"]
+        assert np.array_equal(g["perm"].cpu().numpy(), ref["perm"])
+        assert np.array_equal(g["offsets"].cpu().numpy(), ref["offsets"])
+        us.append(U)
+    us = np.array(us, np.float64)
+    expect = m_prime * (1 - (1 - k / m_prime) ** B)
+    assert abs(us.mean() - expect) <= 4 * us.std(ddof=1) / math.sqrt(draws) + 1e-9
+
+
+def test_zipf_skewed_layers_route_exactly(qwen):
+    shape = qwen.shape
+    B, m_prime = 256, 64
+    x0 = synth.hidden_states(B, shape, 77)
+    ret = synth.retained_set(shape.num_experts, m_prime, 2)
+    us = []
+    for layer_seed in (0, 1):
+        bias = synth.zipf_rank_bias(shape.num_experts, 1.1, 100 + layer_seed)
+        x, wr = synth.apply_popularity_bias(x0, qwen.wr, bias)
+        (_, _), _, route = _case(qwen, B=B, m_prime=m_prime, seed_x=5, seed_imp=2, sample=4, x=x, wr=wr)
+        us.append(int(route["union_size"][0]))
+    # skew concentrates tokens: fewer distinct experts than uniform routing predicts (Sec. 2.1)
+    assert max(us) <= m_prime * (1 - (1 - 8 / m_prime) ** B)
