@@ -1,0 +1,469 @@
+"""Benchmark of the pruned-pool batched-decode MoE layer on GB300.
+
+One step = one decode MoE layer (route/top-k -> group/gather -> expert FFN +
+combine) over one batch of synthetic hidden states, through the C ABI.
+
+Default workload: the Qwen-class layer with the full pool, H=2048, E=128,
+I=768, top-8, decode batch 64 (1.19 GB of touched expert weights per step,
+larger than the 129 MB L2).  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl slimwise|reference]
+                  [--workload qwen_full_b64|qwen_p50_b64|qwen_p50_b128|qwen_p50_b256]
+                  [--sweep] [--stack40]
+
+Under torchrun (N > 1) every rank runs an independent replica of the layer on
+its own GPU (the layer has no cross-GPU exchange); value = tokens of all ranks
+divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_34117_gb300 import synth  # noqa: E402
+
+METRIC = "MoE decode-layer tokens/s; touched-expert HBM GB/s as fraction of ~8 TB/s peak"
+NOMINAL_HBM_GBS = 8000.0
+L2_BYTES = 129 * 1024 * 1024
+WORKLOADS = {
+    "qwen_full_b64": dict(B=64, m_prime=128),
+    "qwen_p50_b64": dict(B=64, m_prime=64),
+    "qwen_p50_b128": dict(B=128, m_prime=64),
+    "qwen_p50_b256": dict(B=256, m_prime=64),
+}
+N_BATCHES = 8  # distinct hidden batches rotated through the timed steps
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------- distributed
+def dist_init():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return ws, rank, local
+
+
+def dist_barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def dist_max(ws, v: float) -> float:
+    if ws <= 1:
+        return v
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(ws, per_rank_tokens: int, per_rank_seconds: float):
+    """(total tokens over ranks, max seconds over ranks)."""
+    return per_rank_tokens * ws, dist_max(ws, per_rank_seconds)
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+        bus = _pci_bus_id(self.idx)
+        if bus:
+            cmd += ["-i", bus]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.reader = threading.Thread(target=self._read, daemon=True)
+            self.reader.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.reader.join(timeout=2)
+        return False
+
+    def summary(self, max_mhz_hint=None):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": max_mhz_hint, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _pci_bus_id(idx):
+    try:
+        p = torch.cuda.get_device_properties(idx)
+        dom, bus, devid = p.pci_domain_id, p.pci_bus_id, p.pci_device_id
+        return f"{dom:08X}:{bus:02X}:{devid:02X}.0"
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------------- inputs
+class LayerInputs:
+    def __init__(self, shape, seed, device, copies=1):
+        self.shape = shape
+        self.copies = []
+        for c in range(copies):
+            w_gu, w_d = synth.expert_weights(shape, seed + 7919 * c, device=device)
+            self.copies.append((w_gu, w_d))
+        self.wr = synth.router_weight(shape, seed, device=device)
+
+    def expert_bytes(self):
+        return self.shape.expert_bytes
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("expert_ffn.cu", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_34117_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """Per-launch DRAM bytes of the expert-FFN kernel from the committed ncu summary,
+    or None when the kernel changed since the capture."""
+    p = os.path.join(ROOT, "profiles", "expert_ffn_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    if d.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    return d.get("per_launch_bytes", {}).get(workload)
+
+
+# ---------------------------------------------------------------- GPU arm
+def run_layer_steps(sw, layer, hidden_batches, retained, k, steps, stream, ws_buf, out, copy_for_step,
+                    ffn_events=None):
+    for i in range(steps):
+        w_gu, w_d = layer.copies[copy_for_step(i)]
+        x = hidden_batches[i % len(hidden_batches)]
+        ev = None if ffn_events is None else ffn_events[i]
+        sw.slimwise_moe_decode_ex(x, layer.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
+                                  stream=stream, ffn_events=ev)
+
+
+def union_sizes(sw, layer, hidden_batches, retained, k):
+    us = []
+    for x in hidden_batches:
+        r = sw.slimwise_moe_route(x, layer.wr, retained, k, layer.shape.num_experts, layer.shape.inter)
+        us.append(int(r["union_size"].item()))
+    return us
+
+
+def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=None):
+    """Time `steps` layer calls; returns a dict of derived numbers."""
+    shape = layer.shape
+    k = shape.top_k
+    batches = [synth.hidden_states(B, shape, seed_x + j, device=device) for j in range(N_BATCHES)]
+    retained = None if m_prime >= shape.num_experts else synth.retained_set(
+        shape.num_experts, m_prime, 2).to(device)
+    ws_buf = sw.alloc_workspace(B, shape.hidden, shape.num_experts, shape.inter, k, device)
+    out = torch.empty((B, shape.hidden), dtype=torch.bfloat16, device=device)
+    us = union_sizes(sw, layer, batches, retained, k)
+    u_mean = float(np.mean(us))
+    touched = u_mean * shape.expert_bytes
+    ncopies = len(layer.copies)
+    rotate = touched < 4 * L2_BYTES and ncopies > 1
+    copy_for_step = (lambda i: i % ncopies) if rotate else (lambda i: 0)
+    stream = torch.cuda.current_stream()
+    run_layer_steps(sw, layer, batches, retained, k, warmup, stream, ws_buf, out, copy_for_step)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    run_layer_steps(sw, layer, batches, retained, k, steps, stream, ws_buf, out, copy_for_step)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    step_ms = t0.elapsed_time(t1) / steps
+    # expert-FFN kernel alone, events on the launch stream
+    ksteps = min(steps, 400)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(ksteps)]
+    run_layer_steps(sw, layer, batches, retained, k, ksteps, stream, ws_buf, out, copy_for_step, ffn_events=evs)
+    torch.cuda.synchronize()
+    ffn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    flags = sw.slimwise_moe_device_status(ws_buf)
+    if flags:
+        raise RuntimeError(f"device error bits {flags:#x}")
+    ffn_bytes = touched + 2 * B * shape.hidden * 2          # union weights + hidden in + out
+    layer_bytes = touched + m_prime * shape.hidden * 4 + 2 * B * shape.hidden * 2
+    return {
+        "B": B, "m_prime": m_prime, "union_mean": u_mean, "union_eq1": m_prime * (1 - (1 - k / m_prime) ** B),
+        "step_ms": step_ms, "tokens_per_s": B / (step_ms * 1e-3),
+        "ffn_ms": ffn_ms, "ffn_algo_bytes": ffn_bytes, "layer_algo_bytes": layer_bytes,
+        "touched_gbs": touched / (step_ms * 1e-3) / 1e9,
+        "ffn_gbs": ffn_bytes / (ffn_ms * 1e-3) / 1e9,
+        "weight_copies_rotated": ncopies if rotate else 1,
+        "_state": (batches, retained, ws_buf, out, copy_for_step),
+    }
+
+
+def e2e_measure(sw, layer, B, m_prime, steps, device, point):
+    """Same metric through the C ABI with host buffers: pinned H2D of the batch,
+    the layer, D2H of the output, all inside the timed region."""
+    shape = layer.shape
+    batches, retained, ws_buf, out, copy_for_step = point["_state"]
+    host_in = [b.cpu().pin_memory() for b in batches]
+    host_out = torch.empty((B, shape.hidden), dtype=torch.bfloat16).pin_memory()
+    dev_in = torch.empty_like(batches[0])
+    stream = torch.cuda.current_stream()
+    k = shape.top_k
+
+    def one(i):
+        dev_in.copy_(host_in[i % len(host_in)], non_blocking=True)
+        w_gu, w_d = layer.copies[copy_for_step(i)]
+        sw.slimwise_moe_decode_ex(dev_in, layer.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
+                                  stream=stream)
+        host_out.copy_(out, non_blocking=True)
+
+    for i in range(5):
+        one(i)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(steps):
+        one(i)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / steps
+    return {"value": B / (ms * 1e-3), "unit": "tokens/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": B * shape.hidden * 2, "d2h_bytes_per_step": B * shape.hidden * 2}
+
+
+def cpu_baseline(layer, B, m_prime, budget_s=15.0):
+    """The CPU oracle as it stands, single-threaded, on a bounded sample of the
+    workload: routing of the whole batch plus the expert FFNs of as many tokens
+    as fit in about `budget_s` seconds.  Returns tokens/s."""
+    import oracle
+    oracle.build()
+    shape = layer.shape
+    w_gu, w_d = layer.copies[0]
+    gu = synth.bf16_bits(w_gu)
+    dn = synth.bf16_bits(w_d)
+    wr = layer.wr.cpu().numpy()
+    x = synth.bf16_bits(synth.hidden_states(B, shape, 1))
+    ret = None if m_prime >= shape.num_experts else synth.retained_set(shape.num_experts, m_prime, 2).numpy()
+    t0 = time.perf_counter()
+    z = oracle.router_logits(x, wr)
+    idx, gates = oracle.route(z, ret, shape.top_k)
+    oracle.group_by_expert(idx, shape.num_experts)
+    t_route = time.perf_counter() - t0
+    n, t_ffn = 0, 0.0
+    while n < B and t_ffn < budget_s:
+        t1 = time.perf_counter()
+        oracle.experts_combine(x, idx, gates, gu, dn, tokens=[n])
+        t_ffn += time.perf_counter() - t1
+        n += 1
+    per_token = t_ffn / n + t_route / B
+    return {"value": 1.0 / per_token, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"routing of all {B} tokens + expert FFNs/combine of {n} tokens of the "
+                      f"{B}-token batch, single thread, {t_route + t_ffn:.1f} s of CPU work",
+            "host_cpus": os.cpu_count()}
+
+
+def main_gpu(args, ws, rank, local):
+    import paper_2609_34117_gb300 as sw
+    from paper_2609_34117_gb300 import build as swbuild
+    if rank == 0 or ws == 1:
+        swbuild.build()
+    dist_barrier(ws)
+    sw.load()
+    device = torch.device("cuda", local)
+    shape = synth.QWEN
+    wl = WORKLOADS[args.workload]
+    B, m_prime = wl["B"], wl["m_prime"]
+    # one weight copy is enough when the touched bytes exceed L2 several times;
+    # the sweep rotates 4 copies for its small-batch points
+    copies = 4 if args.sweep else 1
+    layer = LayerInputs(shape, seed=0, device=device, copies=copies)
+    torch.cuda.synchronize()
+    peak, peak_kind = measured_peaks()
+
+    with ClockSampler(local) as clk:
+        dist_barrier(ws)
+        pt = measure_point(sw, layer, B, m_prime, args.steps, args.warmup, device, seed_x=1)
+        dist_barrier(ws)
+    tokens, secs = aggregate(ws, B * args.steps, pt["step_ms"] * 1e-3 * args.steps)
+    value = tokens / secs
+    e2e = e2e_measure(sw, layer, B, m_prime, min(args.steps, 2000), device, pt)
+    e2e["value"] = e2e["value"] * ws  # replicas: all ranks' tokens
+    achieved = pt["ffn_algo_bytes"] / (pt["ffn_ms"] * 1e-3) / 1e9
+    result = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": pt["step_ms"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
+                   "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B,
+                   "union_mean": pt["union_mean"], "union_eq1": pt["union_eq1"],
+                   "parallelism": f"replicas{ws}",
+                   "l2": "touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
+                         % (pt["union_mean"] * shape.expert_bytes / 1e9)},
+        "touched_hbm": {"gbs": pt["touched_gbs"], "frac_of_8tbs": pt["touched_gbs"] / NOMINAL_HBM_GBS,
+                        "frac_of_measured": pt["touched_gbs"] / peak},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "kernel": "expert_ffn_kernel", "kernel_ms": pt["ffn_ms"],
+                     "algo_bytes_per_launch": pt["ffn_algo_bytes"],
+                     "traffic": profiled_traffic(args.workload)},
+        "e2e": e2e,
+        "gpu_launches": 3 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if args.sweep:
+        result["sweep"] = run_sweep(sw, layer, device, peak)
+    if rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(layer, B, m_prime)
+    elif rank == 0:
+        result["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+def run_sweep(sw, layer, device, peak):
+    pts = []
+    for B in (1, 8, 32, 64, 128, 256, 512):
+        for m_prime in (128, 96, 64, 32):
+            steps = 300 if B <= 64 else 200
+            p = measure_point(sw, layer, B, m_prime, steps, 20, device, seed_x=1000 + B)
+            p.pop("_state")
+            p["touched_frac_of_measured"] = p["touched_gbs"] / peak
+            p["ffn_frac_of_measured"] = p["ffn_gbs"] / peak
+            pts.append(p)
+    return pts
+
+
+# ---------------------------------------------------------------- reference arm
+def main_reference(args, ws, rank):
+    """The reference arm is the CPU oracle, timed as it stands on host cores."""
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    shape = synth.QWEN
+    wl = WORKLOADS[args.workload]
+    B, m_prime = wl["B"], wl["m_prime"]
+    w_gu, w_d = synth.expert_weights(shape, 0)
+    wr = synth.router_weight(shape, 0).numpy()
+    gu, dn = synth.bf16_bits(w_gu), synth.bf16_bits(w_d)
+    ret = None if m_prime >= shape.num_experts else synth.retained_set(shape.num_experts, m_prime, 2).numpy()
+    sample = 4  # tokens whose expert FFNs each step evaluates
+
+    def step(i):
+        x = synth.bf16_bits(synth.hidden_states(B, shape, 1 + (i % N_BATCHES)))
+        t0 = time.perf_counter()
+        z = oracle.router_logits(x, wr)
+        idx, gates = oracle.route(z, ret, shape.top_k)
+        oracle.group_by_expert(idx, shape.num_experts)
+        t_route = time.perf_counter() - t0
+        toks = [(i * sample + j) % B for j in range(sample)]
+        t1 = time.perf_counter()
+        oracle.experts_combine(x, idx, gates, gu, dn, tokens=toks)
+        t_ffn = time.perf_counter() - t1
+        return t_route / B + t_ffn / sample   # seconds per token
+
+    for i in range(args.warmup):
+        step(i)
+    per_tok = [step(i) for i in range(args.steps)]
+    spt = float(np.mean(per_tok))
+    value = 1.0 / spt
+    print(json.dumps({
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": spt * B * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+        "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
+                   "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": f"per step: routing of all {B} tokens + expert FFNs of {sample} tokens, "
+                                   "single thread, scaled to tokens/s"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="slimwise", choices=["slimwise", "reference"])
+    ap.add_argument("--workload", default="qwen_full_b64", choices=sorted(WORKLOADS))
+    ap.add_argument("--sweep", action="store_true", help="batch x pruning sweep (adds 'sweep')")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    ws, rank, local = dist_init()
+    if args.impl == "reference":
+        main_reference(args, ws, rank)
+    else:
+        main_gpu(args, ws, rank, local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
