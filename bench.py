@@ -243,6 +243,10 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     # expert-FFN kernel alone, events on the launch stream
     ksteps = min(steps, 400)
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(ksteps)]
+    for a, b in evs:   # torch creates the CUDA event on its first record
+        a.record(stream)
+        b.record(stream)
+    torch.cuda.synchronize()
     run_layer_steps(sw, layer, batches, retained, k, ksteps, stream, ws_buf, out, copy_for_step, ffn_events=evs)
     torch.cuda.synchronize()
     ffn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))

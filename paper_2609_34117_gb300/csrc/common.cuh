@@ -130,9 +130,20 @@ struct Dims {
 };
 
 // Kernel launch declarations (defined in their own translation units).
+// L2 warm-up issued by the routing kernel while HBM would otherwise idle: the
+// gate/up weights of the first `n_experts` retained experts (in the order of
+// the retained list), which the expert FFN streams first when they are in the
+// batch's union.  A prefetch only moves data into L2; results do not depend on it.
+struct L2Prefetch {
+  const char *base;      // w_gate_up
+  size_t expert_stride;  // bytes from one expert's gate/up block to the next
+  size_t bytes;          // bytes of each expert to prefetch
+  int n_experts;         // 0: no prefetch
+};
+
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
-                              const int32_t *retained, Dims d, Ws ws,
-                              cudaStream_t stream);
+                              const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
+                              bool pdl, cudaStream_t stream);
 cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
                                 bool pdl, bool gather, cudaStream_t stream);
 

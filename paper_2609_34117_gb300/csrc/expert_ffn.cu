@@ -38,16 +38,24 @@ constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange bu
 constexpr int kXchBytes = 2 * kTileRows * kXchStride * 4;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
+// 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
+#ifndef SLIMWISE_STAGE_SUB
+#define SLIMWISE_STAGE_SUB 1
+#endif
+constexpr int kStageSub = SLIMWISE_STAGE_SUB;
+
 struct FfnSmem {
   int stages;
   int stage_bytes;
+  int b_sub_bytes;
   size_t xch_off, bar_off, misc_off, total;
 };
 
 __host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
   FfnSmem p;
   p.stages = stages;
-  p.stage_bytes = kATileBytes + tok_chunk * kBlockK * 2;
+  p.b_sub_bytes = tok_chunk * kBlockK * 2;
+  p.stage_bytes = kStageSub * (kATileBytes + p.b_sub_bytes);
   p.xch_off = (size_t)stages * p.stage_bytes;
   p.bar_off = p.xch_off + kXchBytes;
   // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
@@ -197,7 +205,12 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           slot = 0;
           rphase ^= 1u;
         }
-        if (item >= total) break;
+        if (item >= total) {
+          // no work left for this CTA: the next kernel on the stream may start
+          // its launch (it waits for this grid's completion before reading)
+          pdl_launch_dependents();
+          break;
+        }
         const Item it = decode_item(item, items1, t1, t2, ws);
         if (it.down) {
           // the entry's activations must be complete: all its gate/up tiles
@@ -217,7 +230,8 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           if (!ok) break;
           fence_proxy_async_global();
         }
-        const int nk = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const int nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         const void *amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
         const void *bmap = it.down ? (const void *)&maps.act : (const void *)&maps.xp;
         int row0, row1;
@@ -228,7 +242,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           row0 = it.expert * 2 * d.I + it.tile * kGateRows;
           row1 = row0 + d.I;
         }
-        const uint32_t bytes = (uint32_t)(kATileBytes + it.n16 * kTokBox * kBlockK * 2);
+        const uint32_t sub_bytes = (uint32_t)(kATileBytes + it.n16 * kTokBox * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, kTimeoutNs)) {
@@ -236,14 +250,20 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
             ok = false;
             break;
           }
+          const int nsub = min(kStageSub, nsub_total - kc * kStageSub);
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
-          const uint32_t b = a + kATileBytes;
-          mbar_arrive_expect_tx(full_bar(stage), bytes);
-          tma_load_2d(a, amap, full_bar(stage), kc * kBlockK, row0, pol_w);
-          tma_load_2d(a + kATileBytes / 2, amap, full_bar(stage), kc * kBlockK, row1, pol_w);
-          for (int j = 0; j < it.n16; ++j)
-            tma_load_2d(b + j * (kTokBox * kBlockK * 2), bmap, full_bar(stage),
-                        kc * kBlockK, it.slot_base + j * kTokBox, pol_x);
+          const uint32_t b = a + kStageSub * kATileBytes;
+          mbar_arrive_expect_tx(full_bar(stage), nsub * sub_bytes);
+          for (int s = 0; s < nsub; ++s) {
+            const int x = (kc * kStageSub + s) * kBlockK;
+            const uint32_t as = a + s * kATileBytes;
+            const uint32_t bs = b + s * (uint32_t)plan.b_sub_bytes;
+            tma_load_2d(as, amap, full_bar(stage), x, row0, pol_w);
+            tma_load_2d(as + kATileBytes / 2, amap, full_bar(stage), x, row1, pol_w);
+            for (int j = 0; j < it.n16; ++j)
+              tma_load_2d(bs + j * (kTokBox * kBlockK * 2), bmap, full_bar(stage), x,
+                          it.slot_base + j * kTokBox, pol_x);
+          }
           ++issued;
           if (++stage == stages) {
             stage = 0;
@@ -290,7 +310,8 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(b * nb_cols);
         const uint32_t idesc = idesc_bf16_f32(kTileRows, it.n16 * kTokBox);
-        const int nk = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const int nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(full_bar(stage), phase, abort, kTimeoutNs)) {
@@ -299,13 +320,18 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
             break;
           }
           tc_fence_after();
+          const int nsub = min(kStageSub, nsub_total - kc * kStageSub);
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
-          const uint32_t bb = a + kATileBytes;
+          const uint32_t b = a + kStageSub * kATileBytes;
+          for (int s = 0; s < nsub; ++s) {
+            const uint32_t as = a + s * kATileBytes;
+            const uint32_t bs = b + s * (uint32_t)plan.b_sub_bytes;
 #pragma unroll
-          for (int kk = 0; kk < kBlockK / 16; ++kk)
-            tc_mma_bf16(d_tmem, smem_desc_sw128(a + kk * 32),
-                        smem_desc_sw128(bb + kk * 32), idesc,
-                        (kc | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < kBlockK / 16; ++kk)
+              tc_mma_bf16(d_tmem, smem_desc_sw128(as + kk * 32),
+                          smem_desc_sw128(bs + kk * 32), idesc,
+                          (kc | s | kk) != 0 ? 1u : 0u);
+          }
           tc_commit(empty_bar(stage));
           issued_any = true;
           *consumed = ++n_consumed;

@@ -56,6 +56,7 @@ __global__ void __launch_bounds__(kGroupThreads)
   __shared__ int chunk_cnt[kMaxExperts];
   __shared__ int entry_base[kMaxExperts + 1];
   __shared__ int my_pos[kGroupTokens * kMaxTopK];
+  __shared__ int my_ids[kGroupTokens * kMaxTopK];
   __shared__ int bad;
 
   // Wait for the routing kernel's results; then let the FFN kernel's CTAs
@@ -75,6 +76,7 @@ __global__ void __launch_bounds__(kGroupThreads)
   }
   if (tid == 0) bad = 0;
   __syncthreads();
+  const int nslots = (t1 - t0) * k;
   for (int s = tid; s < S; s += blockDim.x) {
     int e = ws.topk_idx[s];
     if (e < 0 || e >= E) {  // only possible for caller-given selections
@@ -83,34 +85,50 @@ __global__ void __launch_bounds__(kGroupThreads)
     }
     atomicAdd(&cnt_all[e], 1);
     if (s < t0 * k) atomicAdd(&cnt_before[e], 1);
+    else if (s < t1 * k) my_ids[s - t0 * k] = e;
   }
   __syncthreads();
   if (warp == 0) warp_exclusive_scan(cnt_all, offs, E, lane);
   __syncthreads();
 
   // Grouped position of each of this CTA's slots: offset of the expert plus
-  // the number of earlier tokens that selected it.
-  if (tid == 0) {
-    for (int t = t0; t < t1; ++t)
-      for (int j = 0; j < k; ++j) {
-        int e = min(max(ws.topk_idx[t * k + j], 0), E - 1);
-        my_pos[(t - t0) * k + j] = offs[e] + cnt_before[e]++;
-      }
+  // the number of earlier tokens that selected it (tokens before this CTA's
+  // range, then earlier tokens of the range).
+  for (int i = tid; i < nslots; i += blockDim.x) {
+    const int e = my_ids[i];
+    int rank = cnt_before[e];
+    for (int s = 0; s < (i / k) * k; ++s) rank += (my_ids[s] == e) ? 1 : 0;
+    my_pos[i] = offs[e] + rank;
   }
   __syncthreads();
-  const int nslots = (t1 - t0) * k;
   for (int i = tid; i < nslots; i += blockDim.x) {
     const int s = t0 * k + i, p = my_pos[i];
     ws.pos[s] = p;
     ws.perm[p] = s;
   }
   if (do_gather) {
+    // each token row is loaded once into registers and stored to its k
+    // grouped positions; four vectors per thread in flight
     const int vecs = H / 8;  // 16-byte vectors per row
-    for (int i = tid; i < nslots * vecs; i += blockDim.x) {
-      const int r = i / vecs, v = i - r * vecs;
-      const int t = t0 + r / k;
-      reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[r] * H)[v] =
-          reinterpret_cast<const uint4 *>(hidden + (size_t)t * H)[v];
+    const int nt = t1 - t0;
+    constexpr int kVec = 4;
+    for (int i0 = tid; i0 < nt * vecs; i0 += kVec * blockDim.x) {
+      uint4 v[kVec];
+      int tt[kVec], vv[kVec];
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const int i = i0 + u * blockDim.x;
+        tt[u] = i / vecs;
+        vv[u] = i - tt[u] * vecs;
+        if (i < nt * vecs)
+          v[u] = __ldg(reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + tt[u]) * H) + vv[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        if (i0 + u * blockDim.x < nt * vecs)
+          for (int j = 0; j < k; ++j)
+            reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[tt[u] * k + j] * H)[vv[u]] = v[u];
+      }
     }
   }
   const int ht = H / kCombineTile;

@@ -2,22 +2,34 @@
 // renormalised gates (SlimWise Sec. 3.1, Eq. 2 and the renormalisation that
 // follows it).
 //
-// One CTA handles kRouteTokens tokens against every retained expert.  Logits
-// follow the canonical fp32 order: lane l of a warp owns elements
+// A thread-block cluster of kClusterCtas CTAs handles TB tokens.  CTA r of
+// the cluster evaluates the logits of its slice of the retained experts for
+// those tokens and keeps them in its shared memory; after a cluster barrier
+// the warps of CTA 0 run the top-k of each token over all slices, reading the
+// other CTAs' logits through distributed shared memory.  Each CTA thus reads
+// only 1/kClusterCtas of the router rows, and no global counter or second
+// kernel is needed to join the slices.
+//
+// Logits follow the canonical fp32 order: lane l of a warp owns elements
 // 128c + 4l + q (q = 0..3) of every 128-wide chunk c, accumulated with fused
 // multiply-adds in (c, q) order, then the 32 lane partials are combined by an
-// xor butterfly (offsets 16, 8, 4, 2, 1).  The pruned experts are never
+// xor butterfly (offsets 16, 8, 4, 2, 1).  Pruned experts are never
 // evaluated: restricting top-k to K' is the Eq. 2 mask with tau = -inf, with
-// no separate masking pass.  Top-k is a warp-wide arg-max repeated k times
-// on a 64-bit key (order-preserving logit bits, then the complemented expert
+// no separate masking pass.  Top-k is a warp-wide arg-max repeated k times on
+// a 64-bit key (order-preserving logit bits, then the complemented expert
 // id), so ties go to the lowest original id whatever the order of K'.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace slimwise {
 
-constexpr int kRouteTokens = 4;
-constexpr int kRouteThreads = 512;
+constexpr int kRouteThreads = 256;
 constexpr int kRouteWarps = kRouteThreads / 32;
+constexpr int kClusterCtas = 8;
+constexpr int kChunkBatch = 16;  // 128-wide chunks whose loads are issued together
 
 // Order-preserving map of an fp32 value to uint32 (-0 folded onto +0).
 __device__ __forceinline__ uint32_t logit_order_bits(float z) {
@@ -30,25 +42,50 @@ __device__ __forceinline__ float logit_from_order_bits(uint32_t o) {
   return __uint_as_float(b);
 }
 
+template <int TB>
+__device__ __forceinline__ void fma_chunk(const __nv_bfloat16 *xs, int H, int col,
+                                          float4 w, int nt, float (&p)[TB]) {
+#pragma unroll
+  for (int t = 0; t < TB; ++t) {
+    if (t < nt) {
+      const uint2 xr = *reinterpret_cast<const uint2 *>(xs + (size_t)t * H + col);
+      p[t] = fmaf(__uint_as_float(xr.x << 16), w.x, p[t]);
+      p[t] = fmaf(__uint_as_float(xr.x & 0xFFFF0000u), w.y, p[t]);
+      p[t] = fmaf(__uint_as_float(xr.y << 16), w.z, p[t]);
+      p[t] = fmaf(__uint_as_float(xr.y & 0xFFFF0000u), w.w, p[t]);
+    }
+  }
+}
+
+// Shared memory of one CTA: hidden rows [TB][H] bf16, logits of its slice
+// [TB][slice] fp32, retained ids [m] int32.
+template <int TB>
 __global__ void __launch_bounds__(kRouteThreads)
     route_topk_kernel(const __nv_bfloat16 *__restrict__ hidden,
                       const float *__restrict__ router_w,
-                      const int32_t *__restrict__ retained, Dims d, Ws ws) {
+                      const int32_t *__restrict__ retained, Dims d, Ws ws,
+                      L2Prefetch pf) {
   extern __shared__ __align__(16) unsigned char smem[];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int crank = (int)cluster.block_rank();
   const int H = d.H, m = d.m_ret, k = d.k;
+  const int slice = (m + kClusterCtas - 1) / kClusterCtas;
   __nv_bfloat16 *xs = reinterpret_cast<__nv_bfloat16 *>(smem);
-  float *zs = reinterpret_cast<float *>(smem + (size_t)kRouteTokens * H * 2);
-  int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)kRouteTokens * m);
+  float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * 2);
+  int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)TB * slice);
 
+  // The inputs may come from the previous kernel on the stream.
+  pdl_wait_primary();
   // Let the grouping kernel become resident; it waits for this grid to end.
   pdl_launch_dependents();
 
-  const int t0 = blockIdx.x * kRouteTokens;
-  const int nt = min(kRouteTokens, d.B - t0);
+  const int cluster_id = blockIdx.x / kClusterCtas;
+  const int t0 = cluster_id * TB;
+  const int nt = min(TB, d.B - t0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // Retained ids, clamped into [0, E) so a bad id cannot fault; CTA 0 reports
-  // bad and repeated ids and resets the error word of this call.
+  // Retained ids, clamped into [0, E) so a bad id cannot fault; the first CTA
+  // reports bad and repeated ids and resets the error word of this call.
   for (int r = threadIdx.x; r < m; r += blockDim.x) {
     int e = retained ? retained[r] : r;
     ids[r] = min(max(e, 0), d.E - 1);
@@ -73,7 +110,7 @@ __global__ void __launch_bounds__(kRouteThreads)
     if (threadIdx.x == 0) ws.ctrl[kCtrlErr] = bad;
   }
 
-  // Hidden rows of this CTA's tokens (16-byte vectors).
+  // Hidden rows of the cluster's tokens (16-byte vectors).
   const int vecs = H / 8;
   for (int i = threadIdx.x; i < nt * vecs; i += blockDim.x) {
     int t = i / vecs, v = i - t * vecs;
@@ -82,56 +119,69 @@ __global__ void __launch_bounds__(kRouteThreads)
   }
   __syncthreads();
 
-  // Logits: warp per retained expert, all tokens of the CTA at once.
-  for (int r = warp; r < m; r += kRouteWarps) {
-    const float *wrow = router_w + (size_t)ids[r] * H;
-    float p[kRouteTokens];
+  // L2 warm-up: 64 KiB pieces of the first pf.n_experts experts' gate/up
+  // weights, spread over all CTAs of the grid.
+  if (threadIdx.x == 0 && pf.n_experts > 0) {
+    constexpr uint32_t kPiece = 65536;
+    const size_t per_expert = (pf.bytes + kPiece - 1) / kPiece;
+    const size_t pieces = per_expert * (size_t)min(pf.n_experts, m);
+    for (size_t p = blockIdx.x; p < pieces; p += gridDim.x) {
+      const size_t e_i = p / per_expert, off = (p - e_i * per_expert) * kPiece;
+      const uint32_t len = (uint32_t)min((size_t)kPiece, pf.bytes - off);
+      const char *src = pf.base + (size_t)ids[e_i] * pf.expert_stride + off;
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(len) : "memory");
+    }
+  }
+
+  // Logits of this CTA's slice [r_lo, r_hi) of the retained list.
+  const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
+  const int nchunks = H / 128;
+  for (int r = r_lo + warp; r < r_hi; r += kRouteWarps) {
+    const float4 *wrow = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r] * H) + lane;
+    float p[TB];
 #pragma unroll
-    for (int t = 0; t < kRouteTokens; ++t) p[t] = 0.0f;
-#pragma unroll 4
-    for (int c = 0; c < H / 128; ++c) {
-      const float4 w4 = __ldg(reinterpret_cast<const float4 *>(wrow + 128 * c + 4 * lane));
+    for (int t = 0; t < TB; ++t) p[t] = 0.0f;
+    for (int c0 = 0; c0 < nchunks; c0 += kChunkBatch) {
+      float4 v[kChunkBatch];
 #pragma unroll
-      for (int t = 0; t < kRouteTokens; ++t) {
-        if (t < nt) {
-          const uint2 xr = *reinterpret_cast<const uint2 *>(xs + (size_t)t * H + 128 * c + 4 * lane);
-          const float x0 = __uint_as_float(xr.x << 16);
-          const float x1 = __uint_as_float(xr.x & 0xFFFF0000u);
-          const float x2 = __uint_as_float(xr.y << 16);
-          const float x3 = __uint_as_float(xr.y & 0xFFFF0000u);
-          p[t] = fmaf(x0, w4.x, p[t]);
-          p[t] = fmaf(x1, w4.y, p[t]);
-          p[t] = fmaf(x2, w4.z, p[t]);
-          p[t] = fmaf(x3, w4.w, p[t]);
-        }
-      }
+      for (int u = 0; u < kChunkBatch; ++u)
+        if (c0 + u < nchunks) v[u] = __ldg(wrow + 32 * (c0 + u));
+#pragma unroll
+      for (int u = 0; u < kChunkBatch; ++u)
+        if (c0 + u < nchunks) fma_chunk<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v[u], nt, p);
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1)
 #pragma unroll
-      for (int t = 0; t < kRouteTokens; ++t)
-        p[t] = p[t] + __shfl_xor_sync(0xFFFFFFFFu, p[t], off);
+      for (int t = 0; t < TB; ++t) p[t] = p[t] + __shfl_xor_sync(0xFFFFFFFFu, p[t], off);
     if (lane == 0)
 #pragma unroll
-      for (int t = 0; t < kRouteTokens; ++t)
-        if (t < nt) zs[(size_t)t * m + r] = p[t];
+      for (int t = 0; t < TB; ++t)
+        if (t < nt) zs[(size_t)t * slice + (r - r_lo)] = p[t];
   }
-  __syncthreads();
+  cluster.sync();  // every slice's logits are visible cluster-wide
 
-  // Top-k and gates: warp per token.
-  if (warp < nt) {
+  // Top-k and gates: warp w of CTA 0 handles token w of the cluster.
+  if (crank == 0 && warp < nt) {
     const int t = t0 + warp;
-    const float *zt = zs + (size_t)warp * m;
     uint32_t taken = 0;  // bit i: candidate r = lane + 32 i already selected
     float my_z = 0.0f;
     int my_e = 0;
+    // candidate logits of this lane, gathered once from the owning CTAs
+    float cz[kMaxExperts / 32];
+    int nc = 0;
+    for (int r = lane; r < m; r += 32, ++nc) {
+      const int owner = r / slice;
+      const float *zr = cluster.map_shared_rank(zs, owner);
+      cz[nc] = zr[(size_t)warp * slice + (r - owner * slice)];
+    }
     for (int j = 0; j < k; ++j) {
       unsigned long long best = 0ull;
       int i = 0;
       for (int r = lane; r < m; r += 32, ++i) {
         if ((taken >> i) & 1u) continue;
         unsigned long long key =
-            ((unsigned long long)logit_order_bits(zt[r]) << 32) |
+            ((unsigned long long)logit_order_bits(cz[i]) << 32) |
             (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r]);
         best = key > best ? key : best;
       }
@@ -161,24 +211,42 @@ __global__ void __launch_bounds__(kRouteThreads)
       ws.topk_gate[(size_t)t * k + lane] = w / denom;
     }
   }
+  cluster.sync();  // keep every CTA's shared memory alive until CTA 0 is done
 }
 
-size_t route_smem_bytes(const Dims &d) {
-  return (size_t)kRouteTokens * d.H * 2 + (size_t)kRouteTokens * d.m_ret * 4 +
-         (size_t)d.m_ret * 4;
+template <int TB>
+cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
+                            const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
+                            bool pdl, cudaStream_t stream) {
+  const int slice = (d.m_ret + kClusterCtas - 1) / kClusterCtas;
+  const size_t smem = (size_t)TB * d.H * 2 + (size_t)TB * slice * 4 + (size_t)d.m_ret * 4;
+  cudaError_t err = cudaFuncSetAttribute(
+      route_topk_kernel<TB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(((d.B + TB - 1) / TB) * kClusterCtas);
+  cfg.blockDim = dim3(kRouteThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kClusterCtas;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, route_topk_kernel<TB>, hidden, router_w, retained, d, ws, pf);
 }
 
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
-                              const int32_t *retained, Dims d, Ws ws,
-                              cudaStream_t stream) {
-  const size_t smem = route_smem_bytes(d);
-  cudaError_t err = cudaFuncSetAttribute(
-      route_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (err != cudaSuccess) return err;
-  const int grid = (d.B + kRouteTokens - 1) / kRouteTokens;
-  route_topk_kernel<<<grid, kRouteThreads, smem, stream>>>(hidden, router_w,
-                                                           retained, d, ws);
-  return cudaGetLastError();
+                              const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
+                              bool pdl, cudaStream_t stream) {
+  if (d.B <= 32) return launch_route_tb<1>(hidden, router_w, retained, d, ws, pf, pdl, stream);
+  if (d.B <= 64) return launch_route_tb<2>(hidden, router_w, retained, d, ws, pf, pdl, stream);
+  if (d.B <= 256) return launch_route_tb<4>(hidden, router_w, retained, d, ws, pf, pdl, stream);
+  return launch_route_tb<8>(hidden, router_w, retained, d, ws, pf, pdl, stream);
 }
 
 }  // namespace slimwise
