@@ -176,6 +176,29 @@ int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
                        int32_t *union_size, int32_t *perm, int32_t *pos);
 
 /*
+ * slimwise_moe_decode for callers that cannot allocate device memory (an
+ * engine that reserved all of its memory up front, a plugin handed only its
+ * inputs and outputs): the same layer, with the scratch memory taken from a
+ * fixed 16 MiB device array inside this library instead of a caller-given
+ * workspace.  The paper has no counterpart; it is a deployment convenience.
+ *
+ *   Arguments as slimwise_moe_decode, minus workspace / workspace_bytes;
+ *   retained_idx NULL = full pool.
+ *   Limit: slimwise_moe_workspace_size(shape, top_k) must be <= 16 MiB
+ *   (Qwen-class H=2048, E=128, I=768, top-8: B <= 128); larger problems
+ *   return SLIMWISE_ERR_WORKSPACE without launching anything.
+ *   The array's device address is looked up on the first call made on each
+ *   device; make that first call before any stream capture.
+ *   All calls share the array: calls whose kernels may overlap on the GPU
+ *   (unordered streams) race.  No call allocates or frees memory.
+ */
+int slimwise_moe_decode_noalloc(const void *hidden, const float *router_w,
+                                const int32_t *retained_idx, int32_t n_retained,
+                                const void *w_gate_up, const void *w_down,
+                                int32_t top_k, void *out, void *stream,
+                                const slimwise_moe_shape *shape);
+
+/*
  * Reads (and synchronises `stream` for) the device error bits the last call
  * on this workspace left (SLIMWISE_DEVERR_*), writing them to *flags.
  * Returns SLIMWISE_OK if none are set, SLIMWISE_ERR_DEVICE otherwise.

@@ -31,7 +31,7 @@ DEVERR_BAD_TOPK = 0x10
 EXPORTED = (
     "slimwise_status_string", "slimwise_moe_workspace_size", "slimwise_moe_decode",
     "slimwise_moe_decode_full", "slimwise_moe_decode_ex", "slimwise_moe_route",
-    "slimwise_moe_group", "slimwise_moe_device_status",
+    "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
 )
 
 
@@ -76,6 +76,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             lib.slimwise_moe_route.argtypes = [P, P, P, i32, i32, P, SP, P, sz] + [P] * 8
             lib.slimwise_moe_group.argtypes = [P, i32, P, SP, P, sz] + [P] * 6
             lib.slimwise_moe_device_status.argtypes = [P, P, ctypes.POINTER(i32)]
+            lib.slimwise_moe_decode_noalloc.argtypes = [P, P, P, i32, P, P, i32, P, P, SP]
             for name in EXPORTED[1:]:
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
@@ -241,3 +242,27 @@ def slimwise_moe_device_status(workspace, stream=None) -> int:
     if rc not in (0, 5):
         _check(rc, "slimwise_moe_device_status")
     return int(flags.value)
+
+
+def slimwise_moe_decode_noalloc(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
+                                out, stream=None):
+    """The decode layer for callers that cannot allocate device memory.
+
+    The library keeps this entry point's scratch in a fixed 16 MiB device
+    array, so the call needs no workspace; `out` (bf16 [B, H]) must be given.
+    retained_idx None = full pool.  Calls that may overlap on the GPU race on
+    the shared array.
+    """
+    _dev(hidden, torch.bfloat16, "hidden")
+    _dev(router_w, torch.float32, "router_w")
+    _dev(w_gate_up, torch.bfloat16, "w_gate_up")
+    _dev(w_down, torch.bfloat16, "w_down")
+    _dev(out, torch.bfloat16, "out")
+    if retained_idx is not None:
+        _dev(retained_idx, torch.int32, "retained_idx")
+    s = _shape_of(hidden, w_gate_up)
+    n_ret = 0 if retained_idx is None else int(retained_idx.numel())
+    _check(load().slimwise_moe_decode_noalloc(
+        _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),
+        int(top_k), _ptr(out), _stream(stream), ctypes.byref(s)), "slimwise_moe_decode_noalloc")
+    return out

@@ -1,0 +1,67 @@
+// slimwise_noalloc.cu -- decode MoE layer for callers that cannot allocate
+// device memory.
+//
+// Some hosts of this library must not call cudaMalloc or any allocating
+// routine during inference: a serving engine that sized and carved out all
+// of its device memory up front, code that runs under a memory pool or
+// allocator it does not control, or a plugin given only its inputs and
+// outputs.  slimwise_moe_decode_noalloc serves them by running the same three
+// kernels as slimwise_moe_decode with the scratch memory (routing state,
+// grouped activations, expert outputs, counters) placed in a fixed device
+// array that belongs to this library.
+//
+// The array is a file-scope __device__ variable of kNoAllocScratchBytes; every
+// GPU that loads this library holds it until the process exits.  In host code
+// its name is only a host-side stand-in, so its device address is looked up
+// with cudaGetSymbolAddress, once per device, on the first call made with that
+// device current.  That first call should therefore come before any stream
+// capture.  All calls share the array, and it keeps what the last call left
+// there: the kernels set every counter and flag they read at the start of
+// each call, so nothing has to be cleared in between, but two calls whose
+// kernels overlap on the GPU (different streams without ordering) race on it.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace {
+
+// Scratch limit: enough for the Qwen-class layer (H = 2048, E = 128,
+// I = 768, top-8) at decode batches up to 128 tokens.
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[64] = {};
+
+}  // namespace
+
+extern "C" int slimwise_moe_decode_noalloc(const void *hidden, const float *router_w,
+                                           const int32_t *retained_idx, int32_t n_retained,
+                                           const void *w_gate_up, const void *w_down,
+                                           int32_t top_k, void *out, void *stream,
+                                           const slimwise_moe_shape *shape) {
+  if (!shape) return SLIMWISE_ERR_INVALID_ARG;
+  size_t need = 0;
+  int rc = slimwise_moe_workspace_size(shape, top_k, &need);
+  if (rc != SLIMWISE_OK) return rc;
+  // the problem's scratch must fit in the fixed array
+  if (need > kNoAllocScratchBytes) return SLIMWISE_ERR_WORKSPACE;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SLIMWISE_ERR_CUDA;
+  void *scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void *p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+        return SLIMWISE_ERR_CUDA;
+      g_noalloc_ptr[dev] = p;
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  return slimwise_moe_decode_ex(hidden, router_w, retained_idx, n_retained, w_gate_up,
+                                w_down, top_k, out, stream, shape, scratch,
+                                kNoAllocScratchBytes, nullptr);
+}
