@@ -383,8 +383,62 @@ def main_gpu(args, ws, rank, local):
         result["cpu_baseline"] = cpu_baseline(layer, B, m_prime)
     elif rank == 0:
         result["cpu_baseline"] = None
+    if args.stack40:
+        del layer
+        torch.cuda.empty_cache()
+        result["stack40"] = run_stack40(sw, device, max(3, min(args.steps // 100, 20)), 2, peak)
     if rank == 0:
         print(json.dumps(result), flush=True)
+
+
+def run_stack40(sw, device, steps, warmup, peak, n_layers=40, B=256, m_prime=64):
+    """Decode-step MoE stack: n_layers independent Qwen-class layers (own
+    weights, own retained set, own Zipf(1.1) popularity bias), called back to
+    back on one stream; one step = all layers over one batch."""
+    shape = synth.QWEN
+    k = shape.top_k
+    layers = []
+    for l in range(n_layers):
+        w_gu, w_d = synth.expert_weights(shape, 5000 + l, device=device)
+        wr = synth.router_weight(shape, 5000 + l, device=device)
+        bias = synth.zipf_rank_bias(shape.num_experts, 1.1, 9000 + l).to(device)
+        wr[:, -1] = bias
+        ret = synth.retained_set(shape.num_experts, m_prime, 7000 + l).to(device)
+        layers.append((w_gu, w_d, wr, ret))
+    x = synth.hidden_states(B, shape, 1, device=device)
+    x[:, -1] = 1.0
+    ws_buf = sw.alloc_workspace(B, shape.hidden, shape.num_experts, shape.inter, k, device)
+    out = torch.empty((B, shape.hidden), dtype=torch.bfloat16, device=device)
+    us = []
+    for (w_gu, w_d, wr, ret) in layers:
+        r = sw.slimwise_moe_route(x, wr, ret, k, shape.num_experts, shape.inter)
+        us.append(int(r["union_size"].item()))
+    stream = torch.cuda.current_stream()
+
+    def one_step():
+        for (w_gu, w_d, wr, ret) in layers:
+            sw.slimwise_moe_decode_ex(x, wr, ret, w_gu, w_d, k, out=out, workspace=ws_buf, stream=stream)
+
+    for _ in range(warmup):
+        one_step()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(steps):
+        one_step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if sw.slimwise_moe_device_status(ws_buf):
+        raise RuntimeError("device error bits set in the stack run")
+    ms = t0.elapsed_time(t1) / steps
+    touched = sum(us) * shape.expert_bytes
+    return {"layers": n_layers, "B": B, "m_prime": m_prime, "step_ms": ms,
+            "tokens_per_s_through_stack": B / (ms * 1e-3),
+            "layer_tokens_per_s": B * n_layers / (ms * 1e-3),
+            "union_per_layer": us, "union_mean": float(np.mean(us)),
+            "touched_gb_per_step": touched / 1e9, "touched_gbs": touched / (ms * 1e-3) / 1e9,
+            "touched_frac_of_measured": touched / (ms * 1e-3) / 1e9 / peak,
+            "weights_gb": n_layers * shape.num_experts * shape.expert_bytes / 1e9}
 
 
 def run_sweep(sw, layer, device, peak):
@@ -455,6 +509,8 @@ def main():
     ap.add_argument("--impl", default="slimwise", choices=["slimwise", "reference"])
     ap.add_argument("--workload", default="qwen_full_b64", choices=sorted(WORKLOADS))
     ap.add_argument("--sweep", action="store_true", help="batch x pruning sweep (adds 'sweep')")
+    ap.add_argument("--stack40", action="store_true",
+                    help="40 independent skewed layers at m'=64, B=256 (adds 'stack40')")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -42,7 +42,17 @@ enum CtrlWord {
   kCtrlTotalItems = 3,  // gate/up + down work items
   kCtrlWorkCounter = 4, // dynamic scheduler counter
   kCtrlErr = 5,         // SLIMWISE_DEVERR_* bits of the current call
+  kCtrlTraceStep = 6,   // step counter of the optional trace ring
   kCtrlWords = 16
+};
+
+// Optional timeline trace (compile with -DSLIMWISE_TRACE): %globaltimer
+// stamps of each kernel's first CTA, in a ring of kTraceSteps steps that
+// follows the control words.  Without the flag nothing is written.
+constexpr int kTraceSteps = 16;
+enum TraceSlot {
+  kTrRouteStart = 0, kTrRouteEnd, kTrGroupStart, kTrGroupEnd,
+  kTrFfnStart, kTrFfnFirstData, kTrFfnEnd, kTrSlots = 8
 };
 
 // Byte offsets of every workspace region (all 1024-byte aligned).
@@ -67,7 +77,7 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k) {
   };
   const size_t chunk = (size_t)token_chunk_for(B);
   L.max_entries = E + (int32_t)((slots + chunk - 1) / chunk);
-  L.ctrl = take(kCtrlWords * 4);
+  L.ctrl = take(kCtrlWords * 4 + kTraceSteps * kTrSlots * 8);
   L.topk_idx = take(slots * 4);
   L.topk_gate = take(slots * 4);
   L.counts = take((size_t)E * 4);
@@ -170,6 +180,19 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
+}
+
+// Trace stamp of the current step (see TraceSlot); a no-op unless built with
+// SLIMWISE_TRACE.  `step` is the value of ctrl[kCtrlTraceStep] for this call.
+__device__ __forceinline__ void trace_stamp(const Ws &ws, int step, int slot) {
+#ifdef SLIMWISE_TRACE
+  uint64_t *ring = reinterpret_cast<uint64_t *>(ws.ctrl + kCtrlWords);
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  ring[(step & (kTraceSteps - 1)) * kTrSlots + slot] = t;
+#else
+  (void)ws; (void)step; (void)slot;
+#endif
 }
 
 // Programmatic dependent launch.

@@ -31,11 +31,15 @@
 
 namespace slimwise {
 
-constexpr int kFfnThreads = 192;
-constexpr int kEpiThreads = 128;
+constexpr int kEpiGroups = 2;    // epilogue warpgroups, one per TMEM accumulator
+constexpr int kEpiThreads = 128; // threads of one epilogue warpgroup
+constexpr int kFfnThreads = 64 + kEpiGroups * kEpiThreads;
 constexpr int kItemRing = 4;
 constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
-constexpr int kXchBytes = 2 * kTileRows * kXchStride * 4;
+constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
+constexpr int kCombBatch = 16;  // tokens whose combine inputs are staged at once
+// per epilogue group: combine count, token list, staged positions and gates
+constexpr int kGroupMiscInts = 1 + kMaxTokTile + 2 * kCombBatch * kMaxTopK;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 // 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
@@ -60,8 +64,8 @@ __host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
   p.bar_off = p.xch_off + kXchBytes;
   // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
   p.misc_off = p.bar_off + 8 * (2 * stages + 4 + 2 * kItemRing + 1);
-  // item ring, tmem base, abort, consumed stages, combine list count + list
-  p.total = p.misc_off + 4 * (kItemRing + 4) + 4 * kMaxTokTile + 1024;
+  // item ring, tmem base, abort, consumed stages, then per epilogue group
+  p.total = p.misc_off + 4 * (kItemRing + 3) + 4 * kEpiGroups * kGroupMiscInts + 1024;
   return p;
 }
 
@@ -96,8 +100,9 @@ __device__ __forceinline__ Item decode_item(int item, int items1, int t1,
   return it;
 }
 
-__device__ __forceinline__ void epi_bar() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
+// Named barrier of epilogue group g (ids 1.., id 0 is __syncthreads).
+__device__ __forceinline__ void epi_bar(int g) {
+  asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kEpiThreads) : "memory");
 }
 
 __device__ __forceinline__ int ld_acquire(const int *p) {
@@ -134,8 +139,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc + kItemRing);
   volatile int *abort = misc + kItemRing + 1;
   volatile int *consumed = misc + kItemRing + 2;     // stages the MMA finished with
-  int *comb_n = misc + kItemRing + 3;
-  int *comb_list = misc + kItemRing + 4;             // [kMaxTokTile]
+  int *group_misc = misc + kItemRing + 3;            // [kEpiGroups][kGroupMiscInts]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -150,12 +154,11 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     }
     for (int r = 0; r < kItemRing; ++r) {
       mbar_init(itf_bar(r), 1);
-      mbar_init(ite_bar(r), 1 + kEpiThreads);
+      mbar_init(ite_bar(r), 1 + kEpiGroups * kEpiThreads);
     }
     mbar_init(drain_bar, 1);
     *abort = 0;
     *consumed = 0;
-    *comb_n = 0;
     mbar_fence_init();
   }
   if (warp == 0 && lane == 0) {
@@ -175,6 +178,10 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
 
   // Everything below reads the grouping kernel's results.
   pdl_wait_primary();
+#ifdef SLIMWISE_TRACE
+  const int tr_step = ws.ctrl[kCtrlTraceStep] - 1;
+  if (blockIdx.x == 0 && threadIdx.x == 0) trace_stamp(ws, tr_step, kTrFfnStart);
+#endif
 
   const int items1 = __ldcg(&ws.ctrl[kCtrlItems1]);
   const int total = __ldcg(&ws.ctrl[kCtrlTotalItems]);
@@ -320,6 +327,9 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
             break;
           }
           tc_fence_after();
+#ifdef SLIMWISE_TRACE
+          if (blockIdx.x == 0 && n_consumed == 0) trace_stamp(ws, tr_step, kTrFfnFirstData);
+#endif
           const int nsub = min(kStageSub, nsub_total - kc * kStageSub);
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
           const uint32_t b = a + kStageSub * kATileBytes;
@@ -351,9 +361,19 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
+    // Two warpgroups; group g owns TMEM accumulator buffer g, i.e. the items
+    // with local index = g (mod 2), so one group's epilogue overlaps the
+    // other's and the MMA of the next item.
+    const int g = (warp - 2) >> 2;      // epilogue group
     const int q = warp & 3;             // TMEM lane quarter of this warp
     const int row = 32 * q + lane;      // accumulator row = TMEM lane
-    const int et = threadIdx.x - 64;    // 0..127
+    const int et = (threadIdx.x - 64) & (kEpiThreads - 1);
+    float *xb = xch + g * kTileRows * kXchStride;
+    int *gm = group_misc + g * kGroupMiscInts;
+    int *comb_n = gm;
+    int *comb_list = gm + 1;                          // [kMaxTokTile]
+    int *cpos = gm + 1 + kMaxTokTile;                 // [kCombBatch * kMaxTopK]
+    float *cgate = reinterpret_cast<float *>(cpos + kCombBatch * kMaxTopK);
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
@@ -368,8 +388,9 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         rphase ^= 1u;
       }
       if (item >= total) break;
-      const Item it = decode_item(item, items1, t1, t2, ws);
       const int b = local & 1;
+      if (b != g) continue;
+      const Item it = decode_item(item, items1, t1, t2, ws);
       const uint32_t use = (uint32_t)(local >> 1);
       if (!mbar_wait_bounded(accf_bar(b), use & 1u, abort, kTimeoutNs)) {
         if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
@@ -385,10 +406,9 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           uint32_t v[16];
           tmem_ld16(taddr + c * 16, v);
           tmem_ld_wait();
-          float *xb = xch + (c & 1) * kTileRows * kXchStride;
 #pragma unroll
           for (int j = 0; j < 16; ++j) xb[row * kXchStride + j] = __uint_as_float(v[j]);
-          epi_bar();
+          epi_bar(g);
           const int col = c * 16 + n_loc;
           if (col < it.n) {
             uint32_t packed[4];
@@ -397,9 +417,10 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
               float a2[2];
 #pragma unroll
               for (int u2 = 0; u2 < 2; ++u2) {
-                const float g = xb[(i0 + ii + u2) * kXchStride + n_loc];
-                const float u = xb[(kGateRows + i0 + ii + u2) * kXchStride + n_loc];
-                a2[u2] = g / (1.0f + expf(-g)) * u;
+                const float gv = xb[(i0 + ii + u2) * kXchStride + n_loc];
+                const float uv = xb[(kGateRows + i0 + ii + u2) * kXchStride + n_loc];
+                // SiLU(g) * u = g / (1 + e^-g) * u
+                a2[u2] = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
               }
               __nv_bfloat162 h2 = __floats2bfloat162_rn(a2[0], a2[1]);
               packed[ii / 2] = *reinterpret_cast<uint32_t *>(&h2);
@@ -408,13 +429,14 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
                                        it.tile * kGateRows + i0) =
                 make_uint4(packed[0], packed[1], packed[2], packed[3]);
           }
+          epi_bar(g);  // the exchange buffer is rewritten by the next chunk
         }
         tc_fence_before();
         mbar_arrive(acce_bar(b));
         // publish the activations to the TMA (async proxy) readers of any CTA
         fence_proxy_async_global();
         __threadfence();
-        epi_bar();
+        epi_bar(g);
         if (et == 0) atomicAdd(&ws.entry_done[it.entry], 1);
       } else {
         const int h = it.tile * kTileRows + row;
@@ -433,7 +455,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         mbar_arrive(acce_bar(b));
         __threadfence();
         if (et == 0) *comb_n = 0;
-        epi_bar();
+        epi_bar(g);
         // count this contribution for each token; the k-th one combines
         for (int col = et; col < it.n; col += kEpiThreads) {
           const int s = __ldcg(&ws.perm[it.slot_base + col]);
@@ -442,31 +464,68 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           if (old == d.k - 1) comb_list[atomicAdd(comb_n, 1)] = t;
         }
         __threadfence();
-        epi_bar();
+        epi_bar(g);
         const int n_list = *comb_n;
         const int hh = it.tile * kCombineTile + et;
-        for (int i = 0; i < n_list; ++i) {
-          const int t = comb_list[i];
-          float acc = 0.0f;
-          for (int j = 0; j < d.k; ++j) {
-            const int p = __ldcg(&ws.pos[(size_t)t * d.k + j]);
-            const float g = __ldcg(&ws.topk_gate[(size_t)t * d.k + j]);
-            acc = fmaf(g, __ldcg(&ws.y[(size_t)p * d.H + hh]), acc);
+        for (int i0 = 0; i0 < n_list; i0 += kCombBatch) {
+          const int nb = min(kCombBatch, n_list - i0);
+          // stage the grouped positions and gates of this batch of tokens
+          for (int i = et; i < nb * d.k; i += kEpiThreads) {
+            const int t = comb_list[i0 + i / d.k];
+            const int j = i - (i / d.k) * d.k;
+            cpos[i] = __ldcg(&ws.pos[(size_t)t * d.k + j]);
+            cgate[i] = __ldcg(&ws.topk_gate[(size_t)t * d.k + j]);
           }
-          out[(size_t)t * d.H + hh] = __float2bfloat16_rn(acc);
+          epi_bar(g);
+          // out[t, hh] = sum_j g[t,j] y[pos(t,j), hh] in j order; two tokens and
+          // up to eight selections of loads in flight per thread
+          for (int u = 0; u < nb; u += 2) {
+            const bool two = u + 1 < nb;
+            float acc0 = 0.0f, acc1 = 0.0f;
+            for (int j0 = 0; j0 < d.k; j0 += 8) {
+              float v0[8], v1[8];
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) {
+                if (j0 + jj < d.k) {
+                  v0[jj] = __ldcg(&ws.y[(size_t)cpos[u * d.k + j0 + jj] * d.H + hh]);
+                  if (two) v1[jj] = __ldcg(&ws.y[(size_t)cpos[(u + 1) * d.k + j0 + jj] * d.H + hh]);
+                }
+              }
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) {
+                if (j0 + jj < d.k) {
+                  acc0 = fmaf(cgate[u * d.k + j0 + jj], v0[jj], acc0);
+                  if (two) acc1 = fmaf(cgate[(u + 1) * d.k + j0 + jj], v1[jj], acc1);
+                }
+              }
+            }
+            out[(size_t)comb_list[i0 + u] * d.H + hh] = __float2bfloat16_rn(acc0);
+            if (two) out[(size_t)comb_list[i0 + u + 1] * d.H + hh] = __float2bfloat16_rn(acc1);
+          }
+          epi_bar(g);
         }
-        epi_bar();
       }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+#ifdef SLIMWISE_TRACE
+  if (threadIdx.x == 0) {
+    uint64_t t = global_timer_ns();
+    atomicMax(reinterpret_cast<unsigned long long *>(ws.ctrl + kCtrlWords) +
+                  (tr_step & (kTraceSteps - 1)) * kTrSlots + kTrFfnEnd,
+              (unsigned long long)t);
+  }
+#endif
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, (uint32_t)tmem_cols);
   }
 }
+
+// Shared memory kept free next to one FFN CTA (a routing CTA needs ~10 KiB).
+constexpr size_t kCoResidentSmem = 16 * 1024;
 
 int ffn_stages_for(int tok_chunk, size_t smem_limit) {
   int s = 8;
@@ -483,7 +542,9 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   int optin = 0;
   err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (err != cudaSuccess) return err;
-  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin);
+  // leave room on each SM for the next layer's routing CTAs, which become
+  // resident while this grid finishes (programmatic dependent launch)
+  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - kCoResidentSmem);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
   err = cudaFuncSetAttribute(expert_ffn_kernel,

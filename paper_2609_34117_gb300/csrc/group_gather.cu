@@ -63,6 +63,10 @@ __global__ void __launch_bounds__(kGroupThreads)
   // start their prologue.
   pdl_wait_primary();
   pdl_launch_dependents();
+#ifdef SLIMWISE_TRACE
+  const int tr_step = ws.ctrl[kCtrlTraceStep] - 1;
+  if (blockIdx.x == 0 && threadIdx.x == 0) trace_stamp(ws, tr_step, kTrGroupStart);
+#endif
 
   const int B = d.B, k = d.k, E = d.E, H = d.H;
   const int S = B * k;
@@ -173,6 +177,9 @@ __global__ void __launch_bounds__(kGroupThreads)
   }
   __syncthreads();
   if (tid == 0 && bad) atomicOr(&ws.ctrl[kCtrlErr], bad);
+#ifdef SLIMWISE_TRACE
+  if (tid == 0) trace_stamp(ws, tr_step, kTrGroupEnd);
+#endif
 }
 
 cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,

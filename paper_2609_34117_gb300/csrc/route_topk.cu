@@ -29,7 +29,7 @@ namespace slimwise {
 constexpr int kRouteThreads = 256;
 constexpr int kRouteWarps = kRouteThreads / 32;
 constexpr int kClusterCtas = 8;
-constexpr int kChunkBatch = 16;  // 128-wide chunks whose loads are issued together
+constexpr int kChunkBatch = 8;  // 128-wide chunks whose loads are issued together
 
 // Order-preserving map of an fp32 value to uint32 (-0 folded onto +0).
 __device__ __forceinline__ uint32_t logit_order_bits(float z) {
@@ -60,7 +60,9 @@ __device__ __forceinline__ void fma_chunk(const __nv_bfloat16 *xs, int H, int co
 // Shared memory of one CTA: hidden rows [TB][H] bf16, logits of its slice
 // [TB][slice] fp32, retained ids [m] int32.
 template <int TB>
-__global__ void __launch_bounds__(kRouteThreads)
+// Two CTAs per SM worth of registers: a routing CTA must fit beside a
+// persistent expert-FFN CTA so it can be resident before that grid ends.
+__global__ void __launch_bounds__(kRouteThreads, 2)
     route_topk_kernel(const __nv_bfloat16 *__restrict__ hidden,
                       const float *__restrict__ router_w,
                       const int32_t *__restrict__ retained, Dims d, Ws ws,
@@ -78,6 +80,13 @@ __global__ void __launch_bounds__(kRouteThreads)
   pdl_wait_primary();
   // Let the grouping kernel become resident; it waits for this grid to end.
   pdl_launch_dependents();
+#ifdef SLIMWISE_TRACE
+  const int tr_step = ws.ctrl[kCtrlTraceStep];
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    trace_stamp(ws, tr_step, kTrRouteStart);
+    reinterpret_cast<uint64_t *>(ws.ctrl + kCtrlWords)[(tr_step & (kTraceSteps - 1)) * kTrSlots + kTrFfnEnd] = 0;
+  }
+#endif
 
   const int cluster_id = blockIdx.x / kClusterCtas;
   const int t0 = cluster_id * TB;
@@ -212,6 +221,12 @@ __global__ void __launch_bounds__(kRouteThreads)
     }
   }
   cluster.sync();  // keep every CTA's shared memory alive until CTA 0 is done
+#ifdef SLIMWISE_TRACE
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    trace_stamp(ws, tr_step, kTrRouteEnd);
+    ws.ctrl[kCtrlTraceStep] = tr_step + 1;
+  }
+#endif
 }
 
 template <int TB>
