@@ -16,8 +16,9 @@
 // xor butterfly (offsets 16, 8, 4, 2, 1).  Pruned experts are never
 // evaluated: restricting top-k to K' is the Eq. 2 mask with tau = -inf, with
 // no separate masking pass.  Top-k is a warp-wide arg-max repeated k times on
-// a 64-bit key (order-preserving logit bits, then the complemented expert
-// id), so ties go to the lowest original id whatever the order of K'.
+// (order-preserving logit bits desc, expert id asc): each lane sorts its
+// candidates once, then every round is two warp reductions over the lanes'
+// current heads, so ties go to the lowest original id whatever the order of K'.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -93,13 +94,14 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   const int nt = min(TB, d.B - t0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // Retained ids, clamped into [0, E) so a bad id cannot fault; the first CTA
-  // reports bad and repeated ids and resets the error word of this call.
+  // Retained ids, clamped into [0, E) so a bad id cannot fault; the last CTA
+  // (off the critical path of cluster 0's top-k) reports bad and repeated ids
+  // and resets the error word of this call.
   for (int r = threadIdx.x; r < m; r += blockDim.x) {
     int e = retained ? retained[r] : r;
     ids[r] = min(max(e, 0), d.E - 1);
   }
-  if (blockIdx.x == 0) {
+  if (blockIdx.x == gridDim.x - 1) {
     __shared__ uint32_t seen[kMaxExperts / 32];
     __shared__ int bad;
     for (int i = threadIdx.x; i < kMaxExperts / 32; i += blockDim.x) seen[i] = 0;
@@ -173,41 +175,55 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   // Top-k and gates: warp w of CTA 0 handles token w of the cluster.
   if (crank == 0 && warp < nt) {
     const int t = t0 + warp;
-    uint32_t taken = 0;  // bit i: candidate r = lane + 32 i already selected
-    float my_z = 0.0f;
-    int my_e = 0;
-    // candidate logits of this lane, gathered once from the owning CTAs
-    float cz[kMaxExperts / 32];
+    // this lane's candidates r = lane + 32 i as 64-bit keys (order-preserving
+    // logit bits, complemented id), sorted descending; the remote loads of
+    // four candidates are issued before any is used
+    unsigned long long key[kMaxExperts / 32];
     int nc = 0;
-    for (int r = lane; r < m; r += 32, ++nc) {
-      const int owner = r / slice;
-      const float *zr = cluster.map_shared_rank(zs, owner);
-      cz[nc] = zr[(size_t)warp * slice + (r - owner * slice)];
-    }
-    for (int j = 0; j < k; ++j) {
-      unsigned long long best = 0ull;
-      int i = 0;
-      for (int r = lane; r < m; r += 32, ++i) {
-        if ((taken >> i) & 1u) continue;
-        unsigned long long key =
-            ((unsigned long long)logit_order_bits(cz[i]) << 32) |
-            (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r]);
-        best = key > best ? key : best;
+    for (int r0 = lane; r0 < m; r0 += 128) {
+      float zc[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int r = r0 + 32 * u;
+        if (r < m) {
+          const int owner = r / slice;
+          zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
+        }
       }
 #pragma unroll
-      for (int off = 16; off >= 1; off >>= 1) {
-        unsigned long long o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
-        best = o > best ? o : best;
+      for (int u = 0; u < 4; ++u) {
+        const int r = r0 + 32 * u;
+        if (r < m) {
+          const unsigned long long kv = ((unsigned long long)logit_order_bits(zc[u]) << 32) |
+                                        (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r]);
+          int i = nc++;
+          while (i > 0 && key[i - 1] < kv) {
+            key[i] = key[i - 1];
+            --i;
+          }
+          key[i] = kv;
+        }
       }
-      // best == 0 only when fewer than k distinct candidates exist (repeated
-      // retained ids, already reported); fall back to a valid id.
-      const int e_sel = best ? (int)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull)) : ids[0];
-      i = 0;
-      for (int r = lane; r < m; r += 32, ++i)
-        if (ids[r] == e_sel && !((taken >> i) & 1u)) taken |= 1u << i;
+    }
+    // k rounds: the warp's largest head key wins and its lane pops it
+    int head = 0;
+    float my_z = 0.0f;
+    int my_e = 0;
+    for (int j = 0; j < k; ++j) {
+      const unsigned long long mine = head < nc ? key[head] : 0ull;
+      const uint32_t hi = (uint32_t)(mine >> 32), lo = (uint32_t)mine;
+      const uint32_t whi = __reduce_max_sync(0xFFFFFFFFu, hi);
+      const uint32_t wlo = __reduce_max_sync(0xFFFFFFFFu, hi == whi ? lo : 0u);
+      const unsigned long long win = ((unsigned long long)whi << 32) | wlo;
+      // pop every copy of the winner (repeated retained ids give equal keys)
+      while (head < nc && key[head] == win) ++head;
+      uint32_t wid = 0xFFFFFFFFu - wlo;
+      // no candidate left (fewer than k distinct ids, already reported):
+      // fall back to a valid id
+      if (whi == 0u || wid >= (uint32_t)d.E) wid = (uint32_t)ids[0];
       if (lane == j) {
-        my_z = logit_from_order_bits((uint32_t)(best >> 32));
-        my_e = e_sel;
+        my_z = logit_from_order_bits(whi);
+        my_e = (int)wid;
       }
     }
     // g_j = exp(z_j - z_1) / sum_j' exp(z_j' - z_1), the sum in j order.
