@@ -27,12 +27,21 @@ constexpr int kMaxTopK = 32;
 constexpr int kCombineTile = 128;    // h values per down item (= kTileRows)
 
 // Tokens of one expert handled by one work item: the MMA N of the FFN
-// kernel, a multiple of 16 that covers the largest possible per-expert count
-// (B) up to the 256 limit.
-__host__ __device__ inline int token_chunk_for(int B) {
-  int c = (B + 15) / 16 * 16;
-  return c < 16 ? 16 : (c > kMaxTokTile ? kMaxTokTile : c);
+// kernel, a multiple of 16.  It is sized to twice the mean load of a
+// retained expert (B*k/m' selections) rather than to the largest possible
+// load (B): each pipeline stage holds a chunk of token rows, so a smaller
+// chunk leaves room for more weight tiles in flight.  An expert with more
+// tokens than a chunk becomes several entries; their items are handed out
+// together, so the repeated weight reads come from L2.
+__host__ __device__ inline int token_chunk_for(int B, int k, int m_ret) {
+  int most = (B + 15) / 16 * 16;  // an expert is selected at most once per token
+  if (most > kMaxTokTile) most = kMaxTokTile;
+  const int mean = (B * k + m_ret - 1) / m_ret;
+  int c = (2 * mean + 15) / 16 * 16;
+  if (c < 16) c = 16;
+  return c < most ? c : most;
 }
+constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
 
 // Control words at the head of the workspace (int32 each).
 enum CtrlWord {
@@ -75,8 +84,9 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k) {
     o = align_up(o + (bytes ? bytes : 1), 1024);
     return r;
   };
-  const size_t chunk = (size_t)token_chunk_for(B);
-  L.max_entries = E + (int32_t)((slots + chunk - 1) / chunk);
+  // entries: one per selected expert plus one per further chunk; the chunk
+  // size depends on m', so bound it by the smallest chunk
+  L.max_entries = E + (int32_t)((slots + kMinTokChunk - 1) / kMinTokChunk);
   L.ctrl = take(kCtrlWords * 4 + kTraceSteps * kTrSlots * 8);
   L.topk_idx = take(slots * 4);
   L.topk_gate = take(slots * 4);

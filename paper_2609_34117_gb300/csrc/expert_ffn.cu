@@ -528,7 +528,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
 constexpr size_t kCoResidentSmem = 16 * 1024;
 
 int ffn_stages_for(int tok_chunk, size_t smem_limit) {
-  int s = 8;
+  int s = 12;
   while (s > 2 && ffn_smem_plan(tok_chunk, s).total + 1024 > smem_limit) --s;
   return s;
 }

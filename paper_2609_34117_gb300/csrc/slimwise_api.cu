@@ -101,7 +101,7 @@ Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
   d.I = s->inter;
   d.k = top_k;
   d.m_ret = m_ret;
-  d.tok_chunk = token_chunk_for(d.B);
+  d.tok_chunk = token_chunk_for(d.B, top_k, m_ret);
   return d;
 }
 
