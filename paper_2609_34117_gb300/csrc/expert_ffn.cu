@@ -37,9 +37,9 @@ constexpr int kFfnThreads = 64 + kEpiGroups * kEpiThreads;
 constexpr int kItemRing = 4;
 constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
 constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
-constexpr int kCombBatch = 16;  // tokens whose combine inputs are staged at once
-// per epilogue group: combine count, token list, staged positions and gates
-constexpr int kGroupMiscInts = 1 + kMaxTokTile + 2 * kCombBatch * kMaxTopK;
+constexpr int kEpiWarps = kEpiThreads / 32;
+// per epilogue group: combine count and token list
+constexpr int kGroupMiscInts = 1 + kMaxTokTile;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 // 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
@@ -372,8 +372,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     int *gm = group_misc + g * kGroupMiscInts;
     int *comb_n = gm;
     int *comb_list = gm + 1;                          // [kMaxTokTile]
-    int *cpos = gm + 1 + kMaxTokTile;                 // [kCombBatch * kMaxTopK]
-    float *cgate = reinterpret_cast<float *>(cpos + kCombBatch * kMaxTopK);
+    const int ew = q;                                 // warp within the group
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
@@ -466,44 +465,48 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         __threadfence();
         epi_bar(g);
         const int n_list = *comb_n;
-        const int hh = it.tile * kCombineTile + et;
-        for (int i0 = 0; i0 < n_list; i0 += kCombBatch) {
-          const int nb = min(kCombBatch, n_list - i0);
-          // stage the grouped positions and gates of this batch of tokens
-          for (int i = et; i < nb * d.k; i += kEpiThreads) {
-            const int t = comb_list[i0 + i / d.k];
-            const int j = i - (i / d.k) * d.k;
-            cpos[i] = __ldcg(&ws.pos[(size_t)t * d.k + j]);
-            cgate[i] = __ldcg(&ws.topk_gate[(size_t)t * d.k + j]);
+        // out[t, h] = sum_j g[t,j] y[pos(t,j), h] in j order, for the 128 h
+        // of this tile.  A warp takes one token at a time: lane l covers
+        // h = 4l..4l+3 with one 16-byte load per selection (a y tile row is
+        // 512 contiguous bytes), up to 8 loads in flight per lane; lanes
+        // j < k hold selection j's grouped position and gate.
+        const float *ytile = ws.y + it.tile * kCombineTile + 4 * lane;
+        for (int i = ew; i < n_list; i += kEpiWarps) {
+          const int t = comb_list[i];
+          int p = 0;
+          float gj = 0.0f;
+          if (lane < d.k) {
+            p = __ldcg(&ws.pos[(size_t)t * d.k + lane]);
+            gj = __ldcg(&ws.topk_gate[(size_t)t * d.k + lane]);
           }
-          epi_bar(g);
-          // out[t, hh] = sum_j g[t,j] y[pos(t,j), hh] in j order; two tokens and
-          // up to eight selections of loads in flight per thread
-          for (int u = 0; u < nb; u += 2) {
-            const bool two = u + 1 < nb;
-            float acc0 = 0.0f, acc1 = 0.0f;
-            for (int j0 = 0; j0 < d.k; j0 += 8) {
-              float v0[8], v1[8];
+          float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+          for (int j0 = 0; j0 < d.k; j0 += 8) {
+            float4 v[8];
 #pragma unroll
-              for (int jj = 0; jj < 8; ++jj) {
-                if (j0 + jj < d.k) {
-                  v0[jj] = __ldcg(&ws.y[(size_t)cpos[u * d.k + j0 + jj] * d.H + hh]);
-                  if (two) v1[jj] = __ldcg(&ws.y[(size_t)cpos[(u + 1) * d.k + j0 + jj] * d.H + hh]);
-                }
-              }
+            for (int jj = 0; jj < 8; ++jj) {
+              const int pj = __shfl_sync(0xFFFFFFFFu, p, (j0 + jj) & 31);
+              if (j0 + jj < d.k)
+                v[jj] = __ldcg(reinterpret_cast<const float4 *>(ytile + (size_t)pj * d.H));
+            }
 #pragma unroll
-              for (int jj = 0; jj < 8; ++jj) {
-                if (j0 + jj < d.k) {
-                  acc0 = fmaf(cgate[u * d.k + j0 + jj], v0[jj], acc0);
-                  if (two) acc1 = fmaf(cgate[(u + 1) * d.k + j0 + jj], v1[jj], acc1);
-                }
+            for (int jj = 0; jj < 8; ++jj) {
+              const float w = __shfl_sync(0xFFFFFFFFu, gj, (j0 + jj) & 31);
+              if (j0 + jj < d.k) {
+                acc.x = fmaf(w, v[jj].x, acc.x);
+                acc.y = fmaf(w, v[jj].y, acc.y);
+                acc.z = fmaf(w, v[jj].z, acc.z);
+                acc.w = fmaf(w, v[jj].w, acc.w);
               }
             }
-            out[(size_t)comb_list[i0 + u] * d.H + hh] = __float2bfloat16_rn(acc0);
-            if (two) out[(size_t)comb_list[i0 + u + 1] * d.H + hh] = __float2bfloat16_rn(acc1);
           }
-          epi_bar(g);
+          const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
+          const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
+          *reinterpret_cast<uint2 *>(out + (size_t)t * d.H + it.tile * kCombineTile + 4 * lane) =
+              make_uint2(*reinterpret_cast<const uint32_t *>(&lo),
+                         *reinterpret_cast<const uint32_t *>(&hi));
         }
+        // comb_list and comb_n are reused by this group's next down item
+        epi_bar(g);
       }
     }
   }
