@@ -20,26 +20,40 @@ constexpr int kBlockK = 64;          // K elements per pipeline stage (128 B of 
 constexpr int kTileRows = 128;       // MMA M: weight rows per work item
 constexpr int kGateRows = 64;        // gate rows (and as many up rows) per gate/up item
 constexpr int kMaxTokTile = 256;     // MMA N limit: tokens of one expert per item
-constexpr int kTokBox = 16;          // TMA box height for token rows
+constexpr int kTokBox = 16;          // token rows per MMA N step
+constexpr int kTokBoxSizes = 5;      // token-row TMA boxes of kTokBox << m rows, m < 5
 constexpr int kATileBytes = kTileRows * kBlockK * 2;   // 16 KiB
 constexpr int kMaxExperts = 1024;
 constexpr int kMaxTopK = 32;
 constexpr int kCombineTile = 128;    // h values per down item (= kTileRows)
 
-// Tokens of one expert handled by one work item: the MMA N of the FFN
-// kernel, a multiple of 16.  It is sized to twice the mean load of a
-// retained expert (B*k/m' selections) rather than to the largest possible
+// Tokens of one expert handled by one work item (the FFN kernel's largest
+// MMA N): a power of two from 16 to 256, so that one TMA box of a power-of-two
+// height carries an item's token rows.  It is sized to twice the mean load of
+// a retained expert (B*k/m' selections) rather than to the largest possible
 // load (B): each pipeline stage holds a chunk of token rows, so a smaller
 // chunk leaves room for more weight tiles in flight.  An expert with more
 // tokens than a chunk becomes several entries; their items are handed out
 // together, so the repeated weight reads come from L2.
+__host__ __device__ inline int pow2_at_least(int v) {
+  int p = 1;
+  while (p < v) p <<= 1;
+  return p;
+}
 __host__ __device__ inline int token_chunk_for(int B, int k, int m_ret) {
-  int most = (B + 15) / 16 * 16;  // an expert is selected at most once per token
+  int most = pow2_at_least(B);  // an expert is selected at most once per token
+  if (most < kTokBox) most = kTokBox;
   if (most > kMaxTokTile) most = kMaxTokTile;
   const int mean = (B * k + m_ret - 1) / m_ret;
-  int c = (2 * mean + 15) / 16 * 16;
-  if (c < 16) c = 16;
+  int c = pow2_at_least(2 * mean);
+  if (c < kTokBox) c = kTokBox;
   return c < most ? c : most;
+}
+// Index m of the token box (kTokBox << m rows) that covers n16 16-row groups.
+__host__ __device__ inline int token_box_for(int n16) {
+  int m = 0;
+  while ((1 << m) < n16) ++m;
+  return m;
 }
 constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
 
@@ -168,10 +182,10 @@ cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
                                 bool pdl, bool gather, cudaStream_t stream);
 
 struct FfnMaps {
-  CUtensorMap w_gu;   // [E*2I rows, H cols] bf16, box 64 x 64
-  CUtensorMap w_down; // [E*H rows, I cols] bf16, box 64 x 64
-  CUtensorMap xp;     // [B*k rows, H cols] bf16, box 64 x 16
-  CUtensorMap act;    // [B*k rows, I cols] bf16, box 64 x 16
+  CUtensorMap w_gu;                 // [E*2I rows, H cols] bf16, box 64 x 64
+  CUtensorMap w_down;               // [E*H rows, I cols] bf16, box 64 x 64
+  CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16, box 64 x (16 << m)
+  CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16, box 64 x (16 << m)
 };
 
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,

@@ -164,8 +164,10 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&maps.w_gu);
     tma_prefetch_desc(&maps.w_down);
-    tma_prefetch_desc(&maps.xp);
-    tma_prefetch_desc(&maps.act);
+    for (int m = 0; m < kTokBoxSizes && (kTokBox << m) <= d.tok_chunk; ++m) {
+      tma_prefetch_desc(&maps.xp[m]);
+      tma_prefetch_desc(&maps.act[m]);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32((const void *)tmem_slot), (uint32_t)tmem_cols);
@@ -240,7 +242,10 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         const int nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
         const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         const void *amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
-        const void *bmap = it.down ? (const void *)&maps.act : (const void *)&maps.xp;
+        // the item's token rows: one box of the power-of-two height that
+        // covers them (rows past the entry are loaded but not multiplied)
+        const int box_m = token_box_for(it.n16);
+        const void *bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
         int row0, row1;
         if (it.down) {
           row0 = it.expert * d.H + it.tile * kTileRows;
@@ -249,7 +254,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           row0 = it.expert * 2 * d.I + it.tile * kGateRows;
           row1 = row0 + d.I;
         }
-        const uint32_t sub_bytes = (uint32_t)(kATileBytes + it.n16 * kTokBox * kBlockK * 2);
+        const uint32_t sub_bytes = (uint32_t)(kATileBytes + (kTokBox << box_m) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, kTimeoutNs)) {
@@ -267,9 +272,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
             const uint32_t bs = b + s * (uint32_t)plan.b_sub_bytes;
             tma_load_2d(as, amap, full_bar(stage), x, row0, pol_w);
             tma_load_2d(as + kATileBytes / 2, amap, full_bar(stage), x, row1, pol_w);
-            for (int j = 0; j < it.n16; ++j)
-              tma_load_2d(bs + j * (kTokBox * kBlockK * 2), bmap, full_bar(stage), x,
-                          it.slot_base + j * kTokBox, pol_x);
+            tma_load_2d(bs, bmap, full_bar(stage), x, it.slot_base, pol_x);
           }
           ++issued;
           if (++stage == stages) {
@@ -547,6 +550,11 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   if (err != cudaSuccess) return err;
   // leave room on each SM for the next layer's routing CTAs, which become
   // resident while this grid finishes (programmatic dependent launch)
+  // the token maps exist for boxes of 16 << m <= tok_chunk rows, and an
+  // entry's box covers at most tok_chunk rows: tok_chunk must be a power of
+  // two in [16, 256]
+  if (d.tok_chunk < kTokBox || d.tok_chunk > kMaxTokTile || (d.tok_chunk & (d.tok_chunk - 1)))
+    return cudaErrorInvalidValue;
   const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - kCoResidentSmem);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;

@@ -3,6 +3,7 @@
 // decode MoE layer (route/top-k -> group/gather -> expert FFN + combine).
 #include <algorithm>
 #include <cmath>
+#include <cstring>
 #include <mutex>
 
 #include <cudaTypedefs.h>
@@ -134,6 +135,51 @@ int copy_group_outputs(const Ws &w, const Dims &d, cudaStream_t st, int32_t *cou
   return rc;
 }
 
+// The FFN kernel's tensor maps for one call.  Encoding them costs host time
+// on every call, so the maps of the last call on this thread are kept and
+// reused while the pointers and sizes they describe are unchanged.
+struct MapsKey {
+  const void *w_gu, *w_down, *xp, *act;
+  int E, H, I, tok_chunk;
+  uint64_t slots;
+  int device;
+  bool operator==(const MapsKey &o) const {
+    return w_gu == o.w_gu && w_down == o.w_down && xp == o.xp && act == o.act && E == o.E &&
+           H == o.H && I == o.I && tok_chunk == o.tok_chunk && slots == o.slots &&
+           device == o.device;
+  }
+};
+
+bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, const Ws &w,
+                  const Dims &d, uint64_t slots) {
+  thread_local bool have = false;
+  thread_local MapsKey last;
+  thread_local FfnMaps cached;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  const MapsKey key = {w_gate_up, w_down, w.xp, w.act, d.E, d.H, d.I, d.tok_chunk, slots, dev};
+  if (have && key == last) {
+    *maps = cached;
+    return true;
+  }
+  have = false;
+  FfnMaps m;
+  std::memset(&m, 0, sizeof(m));
+  if (encode_map(&m.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
+      encode_map(&m.w_down, w_down, (uint64_t)d.E * d.H, d.I, kGateRows))
+    return false;
+  // token boxes up to the chunk: an item's box covers at most chunk rows
+  for (int b = 0; b < kTokBoxSizes && (kTokBox << b) <= d.tok_chunk; ++b)
+    if (encode_map(&m.xp[b], w.xp, slots, d.H, kTokBox << b) ||
+        encode_map(&m.act[b], w.act, slots, d.I, kTokBox << b))
+      return false;
+  cached = m;
+  last = key;
+  have = true;
+  *maps = m;
+  return true;
+}
+
 int decode_impl(const void *hidden, const float *router_w, const int32_t *retained,
                 int32_t n_retained, const void *w_gate_up, const void *w_down,
                 int32_t top_k, void *out, void *stream, const slimwise_moe_shape *shape,
@@ -162,11 +208,7 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
 
   FfnMaps maps;
   const uint64_t slots = (uint64_t)d.B * d.k;
-  if (encode_map(&maps.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
-      encode_map(&maps.w_down, w_down, (uint64_t)d.E * d.H, d.I, kGateRows) ||
-      encode_map(&maps.xp, w.xp, slots, d.H, kTokBox) ||
-      encode_map(&maps.act, w.act, slots, d.I, kTokBox))
-    return SLIMWISE_ERR_CUDA;
+  if (!ffn_maps_for(&maps, w_gate_up, w_down, w, d, slots)) return SLIMWISE_ERR_CUDA;
 
   // While routing runs, warm L2 with the gate/up weights the FFN streams
   // first -- when the batch almost surely selects every retained expert
