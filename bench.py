@@ -19,6 +19,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -176,10 +177,15 @@ class LayerInputs:
 
 
 def kernel_source_hash():
+    """Hash of the FFN kernel's sources with comments and whitespace removed, so
+    that profiled counters stay attached to the code they were taken on."""
     h = hashlib.sha256()
     for name in ("expert_ffn.cu", "common.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_34117_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2609_34117_gb300", "csrc", name)) as f:
+            src = f.read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", "", src)
+        h.update("".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

@@ -9,12 +9,18 @@
 // tokens as the N operand (16..256, padded to 16) -> TMEM accumulators ->
 // epilogue warps.
 //
-// One persistent CTA per SM (192 threads):
-//   warp 0   producer: takes work items from a global counter, waits for a
-//            down item's activations, issues the TMA loads of each stage.
+// One persistent CTA per SM (320 threads):
+//   warp 0   producer (one thread): takes work items from a global counter,
+//            waits for a down item's activations, and issues each stage's
+//            copies -- the 128-row weight tile (two 64-row boxes) and the
+//            item's token rows (one box, its height the token count rounded
+//            up to a power of two).  The issuing thread's copy rate bounds
+//            the stage rate, so a stage takes three copies whatever the
+//            number of tokens, and the descriptors are chosen once per item.
 //   warp 1   MMA issuer (one thread) and TMEM owner; double-buffered
 //            accumulators so the epilogue of one item overlaps the next.
-//   warps 2-5 epilogue (128 threads, TMEM lane quarters 2,3,0,1).
+//   warps 2-9 two epilogue warpgroups; group g handles the items of
+//            accumulator buffer g (every other item).
 // Work items, all of gate/up before any of down (so a down item only waits
 // for work that has already been handed out):
 //   gate/up (entry, i-tile): A = 64 gate rows + the matching 64 up rows of
