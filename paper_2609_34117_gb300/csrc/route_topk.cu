@@ -43,23 +43,47 @@ __device__ __forceinline__ float logit_from_order_bits(uint32_t o) {
   return __uint_as_float(b);
 }
 
-template <int TB>
-__device__ __forceinline__ void fma_chunk(const __nv_bfloat16 *xs, int H, int col,
-                                          float4 w, int nt, float (&p)[TB]) {
+// Hidden rows are staged in shared memory either as bf16 (half the space) or
+// converted once to fp32 (no per-use conversion: one 16-byte load feeds four
+// multiply-adds).  The product and the summation order are the same.
+__device__ __forceinline__ float4 load_x4(const __nv_bfloat16 *xs, size_t i) {
+  const uint2 xr = *reinterpret_cast<const uint2 *>(xs + i);
+  return make_float4(__uint_as_float(xr.x << 16), __uint_as_float(xr.x & 0xFFFF0000u),
+                     __uint_as_float(xr.y << 16), __uint_as_float(xr.y & 0xFFFF0000u));
+}
+__device__ __forceinline__ float4 load_x4(const float *xs, size_t i) {
+  return *reinterpret_cast<const float4 *>(xs + i);
+}
+
+template <int TB, typename XT>
+__device__ __forceinline__ void fma_chunk(const XT *xs, int H, int col, float4 w,
+                                          float (&p)[TB]) {
 #pragma unroll
   for (int t = 0; t < TB; ++t) {
-    if (t < nt) {
-      const uint2 xr = *reinterpret_cast<const uint2 *>(xs + (size_t)t * H + col);
-      p[t] = fmaf(__uint_as_float(xr.x << 16), w.x, p[t]);
-      p[t] = fmaf(__uint_as_float(xr.x & 0xFFFF0000u), w.y, p[t]);
-      p[t] = fmaf(__uint_as_float(xr.y << 16), w.z, p[t]);
-      p[t] = fmaf(__uint_as_float(xr.y & 0xFFFF0000u), w.w, p[t]);
-    }
+    const float4 x = load_x4(xs, (size_t)t * H + col);
+    p[t] = fmaf(x.x, w.x, p[t]);
+    p[t] = fmaf(x.y, w.y, p[t]);
+    p[t] = fmaf(x.z, w.z, p[t]);
+    p[t] = fmaf(x.w, w.w, p[t]);
   }
 }
 
-// Shared memory of one CTA: hidden rows [TB][H] bf16, logits of its slice
-// [TB][slice] fp32, retained ids [m] int32.
+// Hidden rows are staged as fp32 unless that would keep a routing CTA from
+// fitting beside a persistent expert-FFN CTA (about 20 KiB of shared memory
+// are left there): TB = 4 stays bf16; with TB = 8 no routing CTA fits beside
+// one anyway.
+template <int TB>
+struct StageType {
+  using T = float;
+};
+template <>
+struct StageType<4> {
+  using T = __nv_bfloat16;
+};
+
+// Shared memory of one CTA: hidden rows [TB][H] (StageType), logits of its
+// slice [TB][slice] fp32, retained ids [m] int32.  Rows of tokens past the
+// batch are zero, so every token slot computes (and discards) a logit.
 template <int TB>
 // Two CTAs per SM worth of registers: a routing CTA must fit beside a
 // persistent expert-FFN CTA so it can be resident before that grid ends.
@@ -68,13 +92,14 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
                       const float *__restrict__ router_w,
                       const int32_t *__restrict__ retained, Dims d, Ws ws,
                       L2Prefetch pf) {
+  using XT = typename StageType<TB>::T;
   extern __shared__ __align__(16) unsigned char smem[];
   cg::cluster_group cluster = cg::this_cluster();
   const int crank = (int)cluster.block_rank();
   const int H = d.H, m = d.m_ret, k = d.k;
   const int slice = (m + kClusterCtas - 1) / kClusterCtas;
-  __nv_bfloat16 *xs = reinterpret_cast<__nv_bfloat16 *>(smem);
-  float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * 2);
+  XT *xs = reinterpret_cast<XT *>(smem);
+  float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * sizeof(XT));
   int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)TB * slice);
 
   // The inputs may come from the previous kernel on the stream.
@@ -121,12 +146,22 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
     if (threadIdx.x == 0) ws.ctrl[kCtrlErr] = bad;
   }
 
-  // Hidden rows of the cluster's tokens (16-byte vectors).
+  // Hidden rows of the cluster's tokens (16-byte vectors of 8 bf16), zero
+  // past the batch.
   const int vecs = H / 8;
-  for (int i = threadIdx.x; i < nt * vecs; i += blockDim.x) {
-    int t = i / vecs, v = i - t * vecs;
-    reinterpret_cast<uint4 *>(xs)[(size_t)t * vecs + v] =
-        reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v];
+  for (int i = threadIdx.x; i < TB * vecs; i += blockDim.x) {
+    const int t = i / vecs, v = i - t * vecs;
+    const uint4 raw = t < nt ? reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v]
+                             : make_uint4(0u, 0u, 0u, 0u);
+    if constexpr (sizeof(XT) == 2) {
+      reinterpret_cast<uint4 *>(xs)[(size_t)t * vecs + v] = raw;
+    } else {
+      float4 *dst = reinterpret_cast<float4 *>(xs + (size_t)t * H + 8 * v);
+      dst[0] = make_float4(__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xFFFF0000u),
+                           __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xFFFF0000u));
+      dst[1] = make_float4(__uint_as_float(raw.z << 16), __uint_as_float(raw.z & 0xFFFF0000u),
+                           __uint_as_float(raw.w << 16), __uint_as_float(raw.w & 0xFFFF0000u));
+    }
   }
   __syncthreads();
 
@@ -159,7 +194,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
         if (c0 + u < nchunks) v[u] = __ldg(wrow + 32 * (c0 + u));
 #pragma unroll
       for (int u = 0; u < kChunkBatch; ++u)
-        if (c0 + u < nchunks) fma_chunk<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v[u], nt, p);
+        if (c0 + u < nchunks) fma_chunk<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v[u], p);
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1)
@@ -250,7 +285,8 @@ cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
                             const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
                             bool pdl, cudaStream_t stream) {
   const int slice = (d.m_ret + kClusterCtas - 1) / kClusterCtas;
-  const size_t smem = (size_t)TB * d.H * 2 + (size_t)TB * slice * 4 + (size_t)d.m_ret * 4;
+  const size_t smem = (size_t)TB * d.H * sizeof(typename StageType<TB>::T) +
+                      (size_t)TB * slice * 4 + (size_t)d.m_ret * 4;
   cudaError_t err = cudaFuncSetAttribute(
       route_topk_kernel<TB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
