@@ -39,11 +39,19 @@ from paper_2609_34117_gb300 import synth  # noqa: E402
 METRIC = "MoE decode-layer tokens/s; touched-expert HBM GB/s as fraction of ~8 TB/s peak"
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 1024 * 1024
+SHAPES = {"qwen": synth.QWEN, "qwen36": synth.QWEN36}
 WORKLOADS = {
     "qwen_full_b64": dict(B=64, m_prime=128),
     "qwen_p50_b64": dict(B=64, m_prime=64),
     "qwen_p50_b128": dict(B=128, m_prime=64),
     "qwen_p50_b256": dict(B=256, m_prime=64),
+    # the same 50 % pool as a compact checkpoint holding only the retained
+    # experts (full-pool entry point on [m', ...] tensors)
+    "qwen_compact_p50_b64": dict(B=64, m_prime=64, compact=True),
+    # Qwen3.6-shaped layer (E 256, I 512) at 25 / 50 / 75 % pruning
+    "qwen36_p25_b64": dict(B=64, m_prime=192, shape="qwen36"),
+    "qwen36_p50_b64": dict(B=64, m_prime=128, shape="qwen36"),
+    "qwen36_p75_b64": dict(B=64, m_prime=64, shape="qwen36"),
 }
 N_BATCHES = 8  # distinct hidden batches rotated through the timed steps
 
@@ -172,6 +180,19 @@ class LayerInputs:
             self.copies.append((w_gu, w_d))
         self.wr = synth.router_weight(shape, seed, device=device)
 
+    def compacted(self, m_prime, seed_imp=2):
+        """The layer as a compact checkpoint of its m' retained experts."""
+        from paper_2609_34117_gb300 import checkpoint
+        ret = synth.retained_set(self.shape.num_experts, m_prime, seed_imp).to(self.wr.device)
+        c = LayerInputs.__new__(LayerInputs)
+        c.shape = synth.LayerShape(self.shape.hidden, m_prime, self.shape.inter, self.shape.top_k)
+        c.copies = []
+        for (w_gu, w_d) in self.copies:
+            gu_c, d_c, wr_c, _ = checkpoint.compact_layer(w_gu, w_d, self.wr, ret)
+            c.copies.append((gu_c, d_c))
+        c.wr = wr_c
+        return c
+
     def expert_bytes(self):
         return self.shape.expert_bytes
 
@@ -256,6 +277,20 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     run_layer_steps(sw, layer, batches, retained, k, ksteps, stream, ws_buf, out, copy_for_step, ffn_events=evs)
     torch.cuda.synchronize()
     ffn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    # spread: events around blocks of 10 consecutive layer calls (an event
+    # between every two calls would block the programmatic launch overlap)
+    block = 10
+    nblocks = max(10, min(steps // block, 100))
+    marks = [torch.cuda.Event(enable_timing=True) for _ in range(nblocks + 1)]
+    for ev in marks:
+        ev.record(stream)
+    torch.cuda.synchronize()
+    marks[0].record(stream)
+    for bi in range(nblocks):
+        run_layer_steps(sw, layer, batches, retained, k, block, stream, ws_buf, out, copy_for_step)
+        marks[bi + 1].record(stream)
+    torch.cuda.synchronize()
+    per_step = np.array([marks[i].elapsed_time(marks[i + 1]) / block for i in range(nblocks)])
     flags = sw.slimwise_moe_device_status(ws_buf)
     if flags:
         raise RuntimeError(f"device error bits {flags:#x}")
@@ -268,8 +303,42 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
         "touched_gbs": touched / (step_ms * 1e-3) / 1e9,
         "ffn_gbs": ffn_bytes / (ffn_ms * 1e-3) / 1e9,
         "weight_copies_rotated": ncopies if rotate else 1,
+        "step_ms_p10": float(np.percentile(per_step, 10)),
+        "step_ms_p50": float(np.percentile(per_step, 50)),
+        "step_ms_p90": float(np.percentile(per_step, 90)),
         "_state": (batches, retained, ws_buf, out, copy_for_step),
     }
+
+
+def graph_measure(sw, layer, B, point, calls=20, reps=50):
+    """The same layer calls captured once in a CUDA graph (programmatic launch
+    dependencies become graph edges) and replayed; ms per layer call."""
+    batches, retained, ws_buf, out, copy_for_step = point["_state"]
+    k = layer.shape.top_k
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    try:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(g, stream=side):
+                run_layer_steps(sw, layer, batches, retained, k, calls, side, ws_buf, out, copy_for_step)
+        torch.cuda.current_stream().wait_stream(side)
+        stream = torch.cuda.current_stream()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / (reps * calls)
+        return {"ms_per_step": ms, "tokens_per_s": B / (ms * 1e-3), "calls_per_graph": calls,
+                "replays": reps}
+    except Exception as exc:  # report, do not fail the bench line
+        torch.cuda.synchronize()
+        return {"error": f"{type(exc).__name__}: {exc}"[:200]}
 
 
 def e2e_measure(sw, layer, B, m_prime, steps, device, point):
@@ -343,13 +412,18 @@ def main_gpu(args, ws, rank, local):
     dist_barrier(ws)
     sw.load()
     device = torch.device("cuda", local)
-    shape = synth.QWEN
     wl = WORKLOADS[args.workload]
+    shape = SHAPES[wl.get("shape", "qwen")]
     B, m_prime = wl["B"], wl["m_prime"]
     # one weight copy is enough when the touched bytes exceed L2 several times;
     # the sweep rotates 4 copies for its small-batch points
     copies = 4 if args.sweep else 1
     layer = LayerInputs(shape, seed=0, device=device, copies=copies)
+    sweep_layer = layer
+    if wl.get("compact"):
+        layer = layer.compacted(m_prime)
+        shape = layer.shape
+    torch.cuda.synchronize()
     torch.cuda.synchronize()
     peak, peak_kind = measured_peaks()
 
@@ -359,6 +433,7 @@ def main_gpu(args, ws, rank, local):
         dist_barrier(ws)
     tokens, secs = aggregate(ws, B * args.steps, pt["step_ms"] * 1e-3 * args.steps)
     value = tokens / secs
+    graph = graph_measure(sw, layer, B, pt)
     e2e = e2e_measure(sw, layer, B, m_prime, min(args.steps, 2000), device, pt)
     e2e["value"] = e2e["value"] * ws  # replicas: all ranks' tokens
     achieved = pt["ffn_algo_bytes"] / (pt["ffn_ms"] * 1e-3) / 1e9
@@ -368,6 +443,7 @@ def main_gpu(args, ws, rank, local):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
                    "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B,
+                   "form": "compact checkpoint" if wl.get("compact") else "masked pool",
                    "union_mean": pt["union_mean"], "union_eq1": pt["union_eq1"],
                    "parallelism": f"replicas{ws}",
                    "l2": "touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
@@ -380,11 +456,14 @@ def main_gpu(args, ws, rank, local):
                      "algo_bytes_per_launch": pt["ffn_algo_bytes"],
                      "traffic": profiled_traffic(args.workload)},
         "e2e": e2e,
+        "step_ms_p10_p50_p90": [pt["step_ms_p10"], pt["step_ms_p50"], pt["step_ms_p90"]],
+        "step_spread": "percentiles of the mean step over blocks of 10 consecutive layer calls",
+        "graph": graph,
         "gpu_launches": 3 * args.steps,
         "clocks": clk.summary(),
     }
     if args.sweep:
-        result["sweep"] = run_sweep(sw, layer, device, peak)
+        result["sweep"] = run_sweep(sw, sweep_layer, device, peak)
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(layer, B, m_prime)
     elif rank == 0:
@@ -467,13 +546,19 @@ def main_reference(args, ws, rank):
         return
     import oracle
     oracle.build()
-    shape = synth.QWEN
     wl = WORKLOADS[args.workload]
+    shape = SHAPES[wl.get("shape", "qwen")]
     B, m_prime = wl["B"], wl["m_prime"]
     w_gu, w_d = synth.expert_weights(shape, 0)
     wr = synth.router_weight(shape, 0).numpy()
     gu, dn = synth.bf16_bits(w_gu), synth.bf16_bits(w_d)
     ret = None if m_prime >= shape.num_experts else synth.retained_set(shape.num_experts, m_prime, 2).numpy()
+    if wl.get("compact"):
+        # the retained experts' rows only, in ascending id order
+        ids = np.sort(ret)
+        gu, dn, wr = np.ascontiguousarray(gu[ids]), np.ascontiguousarray(dn[ids]), np.ascontiguousarray(wr[ids])
+        shape = synth.LayerShape(shape.hidden, m_prime, shape.inter, shape.top_k)
+        ret = None
     sample = 4  # tokens whose expert FFNs each step evaluates
 
     def step(i):

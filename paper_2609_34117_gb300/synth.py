@@ -41,6 +41,10 @@ class LayerShape:
 
 TINY = LayerShape(hidden=256, num_experts=16, inter=128, top_k=2)
 QWEN = LayerShape(hidden=2048, num_experts=128, inter=768, top_k=8)
+# Qwen3.6-shaped layer: 256 experts, top-8 (Sec. 2.1).  The expert size is
+# derived, not printed: a 60 GiB bf16 pool over 40 layers of 256 experts is
+# about 3.1 M parameters per expert, i.e. I = 512 at H = 2048.
+QWEN36 = LayerShape(hidden=2048, num_experts=256, inter=512, top_k=8)
 
 
 def _gen(seed: int, device) -> torch.Generator:

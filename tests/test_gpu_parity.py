@@ -57,6 +57,11 @@ def qwen():
     return Layer(synth.QWEN, seed=0)
 
 
+@pytest.fixture(scope="module")
+def qwen36():
+    return Layer(synth.QWEN36, seed=0)
+
+
 def _run(layer, x, retained, k, wr=None, workspace=None):
     wr_d = layer.d_wr if wr is None else wr.to(DEV)
     xd = x.to(DEV)
@@ -161,6 +166,36 @@ def test_qwen_pruned_50pct(qwen, B):
 @pytest.mark.parametrize("B,m_prime", [(1, 128), (8, 96), (32, 32), (128, 96), (512, 32), (512, 128)])
 def test_qwen_sweep_points(qwen, B, m_prime):
     _case(qwen, B=B, m_prime=m_prime, seed_x=1000 + B, seed_imp=2 + m_prime, sample=6)
+
+
+@pytest.mark.parametrize("B,m_prime", [(64, 192), (64, 128), (256, 64), (8, 64)])
+def test_qwen36_shaped_layer(qwen36, B, m_prime):
+    # 256 experts of intermediate size 512: 25 / 50 / 75 % pruning
+    _case(qwen36, B=B, m_prime=m_prime, seed_x=3000 + B, seed_imp=2 + m_prime, sample=6)
+
+
+@pytest.mark.parametrize("m_prime", [64, 32])
+def test_compact_checkpoint_equals_masked_pool(qwen, m_prime):
+    # Sec. 3.1: the Eq. 2 mask over the full pool and a checkpoint holding only
+    # the retained experts give the same layer
+    from paper_2609_34117_gb300 import checkpoint
+    shape = qwen.shape
+    retained = synth.retained_set(shape.num_experts, m_prime, 5, shuffle=True).to(DEV)
+    gu_c, d_c, wr_c, ids = checkpoint.compact_layer(qwen.d_w_gu, qwen.d_w_d, qwen.d_wr, retained)
+    assert gu_c.numel() * shape.num_experts == qwen.d_w_gu.numel() * m_prime
+    x = synth.hidden_states(96, shape, 21).to(DEV)
+    masked = sw.slimwise_moe_decode(x, qwen.d_wr, retained, qwen.d_w_gu, qwen.d_w_d, 8)
+    compact = sw.slimwise_moe_decode_full(x, wr_c, gu_c, d_c, 8)
+    r_m = sw.slimwise_moe_route(x, qwen.d_wr, retained, 8, shape.num_experts, shape.inter)
+    r_c = sw.slimwise_moe_route(x, wr_c, None, 8, m_prime, shape.inter)
+    torch.cuda.synchronize()
+    assert torch.equal(masked, compact)
+    ids_d = ids.to(DEV).long()
+    assert torch.equal(ids_d[r_c["topk_idx"].long()], r_m["topk_idx"].long())
+    assert torch.equal(r_c["topk_gate"], r_m["topk_gate"])
+    assert torch.equal(r_c["perm"], r_m["perm"])
+    assert torch.equal(r_c["counts"], r_m["counts"][ids_d])
+    assert int(r_c["union_size"][0]) == int(r_m["union_size"][0])
 
 
 @pytest.mark.parametrize("B", [1, 5, 17, 33, 300])
