@@ -58,6 +58,8 @@ def _load():
             lib.oracle_expert_swiglu.restype = None
             lib.oracle_experts_combine.argtypes = [P, P, P, P, P, i32, i32, i32, P, i32, P]
             lib.oracle_experts_combine.restype = i32
+            lib.oracle_shared_expert_add.argtypes = [P, P, P, P, i32, i32, P, i32, P, P]
+            lib.oracle_shared_expert_add.restype = i32
             lib.oracle_moe_decode.argtypes = [P, P, P, i32, P, P, i32, i32, i32, i32, i32, P, P, P]
             lib.oracle_moe_decode.restype = i32
             _lib = lib
@@ -159,6 +161,25 @@ def experts_combine(x_bf16, idx, gates, w_gate_up, w_down, tokens=None):
     return out
 
 
+def shared_expert_add(x_bf16, w_shared_gate, w_shared_gu, w_shared_down, out, tokens=None):
+    """Sec. 3.3 shared expert: adds s_t * SE(x_t) to `out` (fp64 [n, H], one row per
+    token of `tokens`) in place; returns the gates s_t (fp64 [n])."""
+    x = _c(x_bf16, np.uint16)
+    wsg = _c(np.asarray(w_shared_gate, np.float32).reshape(-1), np.float32)
+    gu = _c(w_shared_gu, np.uint16)
+    wd = _c(w_shared_down, np.uint16)
+    B, H = x.shape
+    I_s = gu.shape[0] // 2
+    toks = np.arange(B, dtype=np.int32) if tokens is None else _c(np.asarray(tokens, np.int32), np.int32)
+    assert out.dtype == np.float64 and out.flags.c_contiguous and out.shape == (len(toks), H)
+    s = np.empty(len(toks), np.float64)
+    rc = _load().oracle_shared_expert_add(_ptr(x), _ptr(wsg), _ptr(gu), _ptr(wd), H, I_s,
+                                          _ptr(toks), len(toks), _ptr(out), _ptr(s))
+    if rc != 0:
+        raise MemoryError("oracle_shared_expert_add")
+    return s
+
+
 def moe_decode(x_bf16, router_w, retained, w_gate_up, w_down, k):
     """Whole decode layer over the retained pool (retained=None: full pool).
 
@@ -195,6 +216,18 @@ def moe_decode_sampled(x_bf16, router_w, retained, w_gate_up, w_down, k, tokens)
     return {"idx": idx, "gates": gates, "out": out, "z": z}
 
 
+def moe_decode_shared(x_bf16, router_w, retained, w_gate_up, w_down, k, w_shared_gate,
+                      w_shared_gu, w_shared_down, tokens=None):
+    """The layer with its shared expert (Sec. 3.3): routed experts as in
+    `moe_decode`, then s_t * SE(x_t) added.  Expert FFNs for `tokens` only
+    (default: all).  Returns dict(idx, gates, shared_gate, out)."""
+    z = router_logits(x_bf16, router_w)
+    idx, gates = route(z, retained, k)
+    out = experts_combine(x_bf16, idx, gates, w_gate_up, w_down, tokens)
+    s = shared_expert_add(x_bf16, w_shared_gate, w_shared_gu, w_shared_down, out, tokens)
+    return {"idx": idx, "gates": gates, "shared_gate": s, "out": out}
+
+
 # ---------------------------------------------------------------------------
 # Mutation support for the pin suite: compile a modified copy of the oracle
 # source and swap it in, so a test can check that the pins catch a planted
@@ -228,7 +261,8 @@ class swapped_library:
         base = _load()
         lib = ctypes.CDLL(self.path)
         for name in ("oracle_router_logits", "oracle_route", "oracle_group_by_expert",
-                     "oracle_expert_swiglu", "oracle_experts_combine", "oracle_moe_decode"):
+                     "oracle_expert_swiglu", "oracle_experts_combine", "oracle_moe_decode",
+                     "oracle_shared_expert_add"):
             fn_new, fn_old = getattr(lib, name), getattr(base, name)
             fn_new.argtypes, fn_new.restype = fn_old.argtypes, fn_old.restype
         with _lock:

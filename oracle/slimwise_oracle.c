@@ -235,6 +235,44 @@ int oracle_experts_combine(const uint16_t *x, const int32_t *idx,
 }
 
 /*
+ * Shared expert (Sec. 3.3): an always-on SwiGLU expert of intermediate width
+ * I_s, scaled per token by a sigmoid gate.  The distilled layer keeps the
+ * original shared expert and adds a second of the same width under the same
+ * gate, so the deployed form is one expert of twice the width; the oracle
+ * takes whatever width it is given.
+ *   z_t = w_sg . x_t            (canonical fp32 order, as a router logit)
+ *   s_t = 1 / (1 + exp(-z_t))   (fp64)
+ *   out[r, h] += s_t * y^{SE}_h(x_t)        for t = tokens[r]
+ * The shared term is added after the k routed terms.
+ * w_sg: fp32 [H]; w_gu_s: bf16 [2 I_s, H] (gate rows first); w_d_s: bf16
+ * [H, I_s]; out: fp64 [n_tokens, H]; gate_out: fp64 [n_tokens] or NULL.
+ * Returns 0, or -1 on allocation failure.
+ */
+int oracle_shared_expert_add(const uint16_t *x, const float *w_sg,
+                             const uint16_t *w_gu_s, const uint16_t *w_d_s,
+                             int H, int I_s, const int32_t *tokens,
+                             int n_tokens, double *out, double *gate_out) {
+  double *a = (double *)malloc(sizeof(double) * (size_t)(I_s > 0 ? I_s : 1));
+  double *y = (double *)malloc(sizeof(double) * (size_t)H);
+  if (!a || !y) {
+    free(a); free(y);
+    return -1;
+  }
+  for (int r = 0; r < n_tokens; ++r) {
+    int t = tokens[r];
+    float z;
+    oracle_router_logits(x + (size_t)t * H, w_sg, 1, H, 1, &z);
+    double s = 1.0 / (1.0 + exp(-(double)z));
+    if (gate_out) gate_out[r] = s;
+    oracle_expert_swiglu(x + (size_t)t * H, w_gu_s, w_d_s, H, I_s, a, y);
+    double *o = out + (size_t)r * H;
+    for (int h = 0; h < H; ++h) o[h] += s * y[h];
+  }
+  free(a); free(y);
+  return 0;
+}
+
+/*
  * The whole decode MoE layer over the retained pool for every token:
  * logits -> Eq. 2 mask -> top-k -> renormalised gates -> expert FFNs ->
  * gate-weighted combine.  retained = NULL means the full pool.

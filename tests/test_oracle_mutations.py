@@ -29,6 +29,10 @@ MUTATIONS = {
                         "acc += (double)bf16_to_float(wd[(size_t)i * H + h]) * a[i];"),
     # combine: gates not applied
     "combine_no_gate": ("for (int h = 0; h < H; ++h) o[h] += g * y[h];", "for (int h = 0; h < H; ++h) o[h] += y[h];"),
+    # shared expert: sigmoid with the wrong sign
+    "shared_gate_sign": ("double s = 1.0 / (1.0 + exp(-(double)z));", "double s = 1.0 / (1.0 + exp((double)z));"),
+    # shared expert: gate not applied
+    "shared_gate_dropped": ("for (int h = 0; h < H; ++h) o[h] += s * y[h];", "for (int h = 0; h < H; ++h) o[h] += y[h];"),
     # grouping: offsets off by one expert
     "offsets_shift": ("offsets[e + 1] = offsets[e] + counts[e];", "offsets[e + 1] = offsets[e] + counts[e > 0 ? e - 1 : 0];"),
     # grouping: token order reversed inside an expert
@@ -46,6 +50,9 @@ PIN_FUNCS = [
     (pins.test_top1_one_hot_router_is_dense_ffn, ()),
     (pins.test_closed_form_selection_experts_and_gates, ()),
     (pins.test_grouping_structure_and_stable_sort, (33, 8, 128)),
+    (pins.test_shared_expert_gate_is_sigmoid_of_canonical_logit, ()),
+    (pins.test_shared_expert_saturated_gates, ()),
+    (pins.test_shared_expert_twice_width_is_sum_of_halves, ()),
 ]
 
 

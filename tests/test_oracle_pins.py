@@ -299,3 +299,80 @@ def test_union_size_matches_eq1_expectation(oracle_lib, m_prime, B):
     expect = m_prime * (1.0 - (1.0 - k / m_prime) ** B)
     sem = max(u.std(ddof=1), 1e-9) / math.sqrt(draws)
     assert abs(u.mean() - expect) <= 4 * sem + 1e-9, (u.mean(), expect, sem)
+
+
+# --------------------------------------------------------------------------
+# Shared expert (Sec. 3.3): always-on SwiGLU expert under a sigmoid gate
+# --------------------------------------------------------------------------
+def _shared_expert(seed, I_s, H=256):
+    one = synth.LayerShape(hidden=H, num_experts=1, inter=I_s, top_k=1)
+    gu, dn = synth.expert_weights(one, seed)
+    g = torch.Generator().manual_seed(seed + 17)
+    w_sg = (torch.randn(H, generator=g) * 0.05).to(torch.float32)
+    return _bits(gu[0]), _bits(dn[0]), w_sg.numpy()
+
+
+def _shared_only(oracle_lib, xb, w_sg, gu, dn):
+    out = np.zeros((xb.shape[0], xb.shape[1]), np.float64)
+    s = oracle_lib.shared_expert_add(xb, w_sg, gu, dn, out)
+    return out, s
+
+
+def test_shared_expert_gate_is_sigmoid_of_canonical_logit(oracle_lib):
+    x, _, _, _ = _tiny_layer(B=5)
+    xb = _bits(x)
+    gu, dn, w_sg = _shared_expert(3, 64)
+    _, s = _shared_only(oracle_lib, xb, w_sg, gu, dn)
+    x64 = _bf16_to_f64(xb)
+    z_exact = x64 @ w_sg.astype(np.float64)
+    absdot = np.abs(x64) @ np.abs(w_sg.astype(np.float64))
+    n_ops = xb.shape[1] // 32 + 5
+    gamma = n_ops * 2.0 ** -24 / (1 - n_ops * 2.0 ** -24)
+    # |ds/dz| <= 1/4: the gate is the sigmoid of z within the fp32 sum's error
+    ref = 1.0 / (1.0 + np.exp(-z_exact))
+    assert np.all(np.abs(s - ref) <= 0.25 * gamma * absdot + 1e-15)
+    assert np.all((s > 0) & (s < 1))
+
+
+def test_shared_expert_saturated_gates(oracle_lib):
+    # gate logit -1000: the shared term vanishes exactly; +1000: the whole
+    # expert is added, equal to a dense numpy SwiGLU
+    shape = synth.TINY
+    x, wr, w_gu, w_d = _tiny_layer(B=4)
+    x, wr = synth.apply_popularity_bias(x, wr, torch.zeros(shape.num_experts))
+    xb, w, gu_r, dn_r = _bits(x), wr.numpy(), _bits(w_gu), _bits(w_d)
+    retained = synth.retained_set(shape.num_experts, 8, seed=2).numpy()
+    gu, dn, w_sg = _shared_expert(5, 64)
+    w_sg = np.zeros_like(w_sg)
+    routed = oracle_lib.moe_decode(xb, w, retained, gu_r, dn_r, 2)["out"]
+    w_sg[-1] = -1000.0
+    off = oracle_lib.moe_decode_shared(xb, w, retained, gu_r, dn_r, 2, w_sg, gu, dn)
+    assert np.all(off["shared_gate"] == 0.0)
+    assert np.array_equal(off["out"], routed)
+    w_sg[-1] = 1000.0
+    on = oracle_lib.moe_decode_shared(xb, w, retained, gu_r, dn_r, 2, w_sg, gu, dn)
+    assert np.all(on["shared_gate"] == 1.0)
+    x64 = _bf16_to_f64(xb)
+    dense = np.stack([_dense_swiglu(x64[t], _bf16_to_f64(gu), _bf16_to_f64(dn)) for t in range(4)])
+    np.testing.assert_allclose(on["out"] - routed, dense, rtol=1e-9, atol=1e-12)
+
+
+def test_shared_expert_twice_width_is_sum_of_halves(oracle_lib):
+    # Sec. 3.3: two shared experts under one gate are one expert of twice the
+    # intermediate width ([gate1; gate2; up1; up2] rows, [down1 | down2] columns)
+    x, _, _, _ = _tiny_layer(B=3)
+    xb = _bits(x)
+    gu1, dn1, w_sg = _shared_expert(7, 32)
+    gu2, dn2, _ = _shared_expert(8, 32)
+    I = 32
+    gu = np.concatenate([gu1[:I], gu2[:I], gu1[I:], gu2[I:]], axis=0)
+    dn = np.concatenate([dn1, dn2], axis=1)
+    both, s = _shared_only(oracle_lib, xb, w_sg, gu, dn)
+    a, _ = _shared_only(oracle_lib, xb, w_sg, gu1, dn1)
+    b, _ = _shared_only(oracle_lib, xb, w_sg, gu2, dn2)
+    np.testing.assert_allclose(both, a + b, rtol=1e-12, atol=1e-15)
+    # the second expert starts with a zero down projection: the layer output
+    # is unchanged at initialisation
+    dn_init = np.concatenate([dn1, np.zeros_like(dn2)], axis=1)
+    init, _ = _shared_only(oracle_lib, xb, w_sg, gu, dn_init)
+    assert np.array_equal(init, a)
