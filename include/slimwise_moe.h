@@ -176,6 +176,38 @@ int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
                        int32_t *union_size, int32_t *perm, int32_t *pos);
 
 /*
+ * The decode layer with a shared expert (Sec. 3.3): an always-on SwiGLU
+ * expert of intermediate width Is under a per-token sigmoid gate, added after
+ * the k routed experts.  Qwen3.6's distilled decoder keeps its original
+ * shared expert and a second one of the same width under the same gate, i.e.
+ * one shared expert of twice the width, which is what this call takes.
+ *
+ *   out[t] = sum_j g[t,j] E_{idx[t,j]}(x_t) + s_t * SE(x_t)
+ *   s_t    = 1 / (1 + exp(-w_shared_gate . x_t)) (fp32; the dot product in
+ *            the same summation order as the router logits)
+ *
+ *   w_shared_gate    fp32 [H]        gate row, 16-byte aligned
+ *   w_shared_gate_up bf16 [2Is, H]   rows [0, Is) = gate, [Is, 2Is) = up
+ *   w_shared_down    bf16 [H, Is]
+ *   inter_shared     Is, a multiple of 64 in [64, 65536]
+ *   workspace        >= slimwise_moe_shared_workspace_size() bytes
+ * Other arguments as slimwise_moe_decode; retained_idx NULL = full pool.
+ * Errors as slimwise_moe_decode; a bad Is or a misaligned shared pointer
+ * returns SLIMWISE_ERR_UNSUPPORTED_SHAPE, a NULL one SLIMWISE_ERR_INVALID_ARG.
+ */
+int slimwise_moe_shared_workspace_size(const slimwise_moe_shape *shape, int32_t top_k,
+                                       int32_t inter_shared, size_t *bytes);
+int slimwise_moe_decode_shared(const void *hidden, const float *router_w,
+                               const int32_t *retained_idx, int32_t n_retained,
+                               const void *w_gate_up, const void *w_down,
+                               int32_t top_k, const float *w_shared_gate,
+                               const void *w_shared_gate_up,
+                               const void *w_shared_down, int32_t inter_shared,
+                               void *out, void *stream,
+                               const slimwise_moe_shape *shape, void *workspace,
+                               size_t workspace_bytes);
+
+/*
  * slimwise_moe_decode for callers that cannot allocate device memory (an
  * engine that reserved all of its memory up front, a plugin handed only its
  * inputs and outputs): the same layer, with the scratch memory taken from a
@@ -185,7 +217,7 @@ int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
  *   Arguments as slimwise_moe_decode, minus workspace / workspace_bytes;
  *   retained_idx NULL = full pool.
  *   Limit: slimwise_moe_workspace_size(shape, top_k) must be <= 16 MiB
- *   (Qwen-class H=2048, E=128, I=768, top-8: B <= 128); larger problems
+ *   (Qwen-class H=2048, E=128, I=768, top-8: B <= 151); larger problems
  *   return SLIMWISE_ERR_WORKSPACE without launching anything.
  *   The array's device address is looked up on the first call made on each
  *   device; make that first call before any stream capture.

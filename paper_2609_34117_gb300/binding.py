@@ -32,6 +32,7 @@ EXPORTED = (
     "slimwise_status_string", "slimwise_moe_workspace_size", "slimwise_moe_decode",
     "slimwise_moe_decode_full", "slimwise_moe_decode_ex", "slimwise_moe_route",
     "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
+    "slimwise_moe_shared_workspace_size", "slimwise_moe_decode_shared",
 )
 
 
@@ -77,6 +78,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
             lib.slimwise_moe_group.argtypes = [P, i32, P, SP, P, sz] + [P] * 6
             lib.slimwise_moe_device_status.argtypes = [P, P, ctypes.POINTER(i32)]
             lib.slimwise_moe_decode_noalloc.argtypes = [P, P, P, i32, P, P, i32, P, P, SP]
+            lib.slimwise_moe_shared_workspace_size.argtypes = [SP, i32, i32, ctypes.POINTER(sz)]
+            lib.slimwise_moe_decode_shared.argtypes = [P, P, P, i32, P, P, i32, P, P, P, i32,
+                                                       P, P, SP, P, sz]
             for name in EXPORTED[1:]:
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
@@ -141,6 +145,49 @@ def _prep(hidden, router_w, w_gate_up, w_down, top_k, out, workspace):
         workspace = alloc_workspace(s.num_tokens, s.hidden, s.num_experts, s.inter, top_k,
                                     hidden.device)
     return s, out, workspace
+
+
+def slimwise_moe_shared_workspace_size(num_tokens: int, hidden: int, num_experts: int, inter: int,
+                                       top_k: int, inter_shared: int) -> int:
+    out = ctypes.c_size_t(0)
+    s = Shape(num_tokens, hidden, num_experts, inter)
+    _check(load().slimwise_moe_shared_workspace_size(ctypes.byref(s), top_k, int(inter_shared),
+                                                     ctypes.byref(out)),
+           "slimwise_moe_shared_workspace_size")
+    return int(out.value)
+
+
+def slimwise_moe_decode_shared(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
+                               w_shared_gate, w_shared_gate_up, w_shared_down, out=None,
+                               workspace=None, stream=None):
+    """Decode MoE layer with a shared expert under a sigmoid gate (Sec. 3.3);
+    retained_idx None = full pool.  Returns `out`."""
+    _dev(hidden, torch.bfloat16, "hidden")
+    _dev(router_w, torch.float32, "router_w")
+    _dev(w_gate_up, torch.bfloat16, "w_gate_up")
+    _dev(w_down, torch.bfloat16, "w_down")
+    _dev(w_shared_gate, torch.float32, "w_shared_gate")
+    _dev(w_shared_gate_up, torch.bfloat16, "w_shared_gate_up")
+    _dev(w_shared_down, torch.bfloat16, "w_shared_down")
+    s = _shape_of(hidden, w_gate_up)
+    inter_shared = int(w_shared_gate_up.shape[0]) // 2
+    if out is None:
+        out = torch.empty((s.num_tokens, s.hidden), dtype=torch.bfloat16, device=hidden.device)
+    _dev(out, torch.bfloat16, "out")
+    if workspace is None:
+        n = slimwise_moe_shared_workspace_size(s.num_tokens, s.hidden, s.num_experts, s.inter,
+                                               top_k, inter_shared)
+        workspace = torch.empty(n, dtype=torch.uint8, device=hidden.device)
+    n_ret = 0
+    if retained_idx is not None:
+        _dev(retained_idx, torch.int32, "retained_idx")
+        n_ret = int(retained_idx.numel())
+    _check(load().slimwise_moe_decode_shared(
+        _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),
+        int(top_k), _ptr(w_shared_gate), _ptr(w_shared_gate_up), _ptr(w_shared_down),
+        inter_shared, _ptr(out), _stream(stream), ctypes.byref(s), _ptr(workspace),
+        workspace.numel()), "slimwise_moe_decode_shared")
+    return out
 
 
 def slimwise_moe_decode(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,

@@ -61,8 +61,8 @@ constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the e
 enum CtrlWord {
   kCtrlUnionSize = 0,
   kCtrlNumEntries = 1,
-  kCtrlItems1 = 2,      // gate/up work items
-  kCtrlTotalItems = 3,  // gate/up + down work items
+  kCtrlItems1 = 2,      // routed gate/up work items
+  kCtrlTotalItems = 3,  // all work items (shared and routed, gate/up and down)
   kCtrlWorkCounter = 4, // dynamic scheduler counter
   kCtrlErr = 5,         // SLIMWISE_DEVERR_* bits of the current call
   kCtrlTraceStep = 6,   // step counter of the optional trace ring
@@ -81,7 +81,7 @@ enum TraceSlot {
 // Byte offsets of every workspace region (all 1024-byte aligned).
 struct WsLayout {
   size_t ctrl, topk_idx, topk_gate, counts, offsets, union_ids, entries,
-      entry_done, perm, pos, comb_cnt, xp, act, y, total;
+      entry_done, perm, pos, comb_cnt, xp, act, y, shared_gate, xt, act_s, y_s, total;
   int32_t max_entries;
 };
 
@@ -89,7 +89,8 @@ __host__ __device__ inline size_t align_up(size_t v, size_t a) {
   return (v + a - 1) / a * a;
 }
 
-inline WsLayout make_layout(int B, int H, int E, int I, int k) {
+// Is: intermediate width of the shared expert (0: none).
+inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
   WsLayout L;
   size_t o = 0;
   const size_t slots = (size_t)B * k;
@@ -99,8 +100,10 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k) {
     return r;
   };
   // entries: one per selected expert plus one per further chunk; the chunk
-  // size depends on m', so bound it by the smallest chunk
-  L.max_entries = E + (int32_t)((slots + kMinTokChunk - 1) / kMinTokChunk);
+  // size depends on m', so bound it by the smallest chunk; the shared expert
+  // adds one entry per chunk of the batch
+  L.max_entries = E + (int32_t)((slots + kMinTokChunk - 1) / kMinTokChunk) +
+                  (Is > 0 ? (B + kMinTokChunk - 1) / kMinTokChunk : 0);
   L.ctrl = take(kCtrlWords * 4 + kTraceSteps * kTrSlots * 8);
   L.topk_idx = take(slots * 4);
   L.topk_gate = take(slots * 4);
@@ -115,6 +118,14 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k) {
   L.xp = take(slots * H * 2);
   L.act = take(slots * I * 2);
   L.y = take(slots * H * 4);
+  if (Is > 0) {
+    L.shared_gate = take((size_t)B * 4);
+    L.xt = take((size_t)B * H * 2);
+    L.act_s = take((size_t)B * Is * 2);
+    L.y_s = take((size_t)B * H * 4);
+  } else {  // no shared expert: no space (these regions are never accessed)
+    L.shared_gate = L.xt = L.act_s = L.y_s = o;
+  }
   L.total = o;
   return L;
 }
@@ -135,6 +146,10 @@ struct Ws {
   __nv_bfloat16 *xp;   // [B*k, H] hidden rows in grouped order
   __nv_bfloat16 *act;  // [B*k, I] SwiGLU activations in grouped order
   float *y;            // [B*k, H] expert outputs in grouped order
+  float *shared_gate;  // [B] sigmoid gate of the shared expert
+  __nv_bfloat16 *xt;   // [B, H] hidden rows, token order (shared-expert input)
+  __nv_bfloat16 *act_s;  // [B, Is] shared-expert activations, token order
+  float *y_s;          // [B, H] shared-expert outputs, token order
 };
 
 inline Ws make_ws(void *base, const WsLayout &L) {
@@ -154,13 +169,19 @@ inline Ws make_ws(void *base, const WsLayout &L) {
   w.xp = (__nv_bfloat16 *)(b + L.xp);
   w.act = (__nv_bfloat16 *)(b + L.act);
   w.y = (float *)(b + L.y);
+  w.shared_gate = (float *)(b + L.shared_gate);
+  w.xt = (__nv_bfloat16 *)(b + L.xt);
+  w.act_s = (__nv_bfloat16 *)(b + L.act_s);
+  w.y_s = (float *)(b + L.y_s);
   return w;
 }
 
 struct Dims {
   int B, H, E, I, k;
   int m_ret;      // retained experts (E for the full pool)
-  int tok_chunk;  // max tokens of one expert per work item (multiple of 16, <= 256)
+  int tok_chunk;  // max tokens of one expert per work item (power of two, 16..256)
+  int Is;         // shared-expert intermediate width (0: no shared expert)
+  int S;          // shared-expert work entries: ceil(B / tok_chunk), 0 without one
 };
 
 // Kernel launch declarations (defined in their own translation units).
@@ -178,14 +199,20 @@ struct L2Prefetch {
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
                               const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
                               bool pdl, cudaStream_t stream);
-cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
-                                bool pdl, bool gather, cudaStream_t stream);
+// w_shared_gate: fp32 [H] gate row of the shared expert, or NULL (d.Is == 0).
+cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shared_gate,
+                                Dims d, Ws ws, bool pdl, bool gather, cudaStream_t stream);
 
 struct FfnMaps {
   CUtensorMap w_gu;                 // [E*2I rows, H cols] bf16, box 64 x 64
   CUtensorMap w_down;               // [E*H rows, I cols] bf16, box 64 x 64
   CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16, box 64 x (16 << m)
   CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16, box 64 x (16 << m)
+  // shared expert (encoded only when there is one)
+  CUtensorMap w_gu_s;               // [2Is rows, H cols] bf16, box 64 x 64
+  CUtensorMap w_down_s;             // [H rows, Is cols] bf16, box 64 x 64
+  CUtensorMap xt[kTokBoxSizes];     // [B rows, H cols] bf16, hidden in token order
+  CUtensorMap act_s[kTokBoxSizes];  // [B rows, Is cols] bf16, token order
 };
 
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,

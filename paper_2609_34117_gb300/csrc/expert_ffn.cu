@@ -77,6 +77,7 @@ __host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
 
 struct Item {
   int down;      // 0: gate/up, 1: down
+  int shared;    // 1: the shared expert (token order), 0: a routed expert
   int entry;
   int tile;
   int expert;
@@ -85,18 +86,48 @@ struct Item {
   int n16;       // tokens rounded up to 16, / 16
 };
 
-__device__ __forceinline__ Item decode_item(int item, int items1, int t1,
-                                            int t2, const Ws &ws) {
+// Work-item ranges of one launch, in the order they are handed out:
+//   [shared gate/up: S*t1s][routed gate/up: r1][shared down: S*t2][routed down]
+// Every gate/up item precedes every down item; the shared expert's items go
+// first in each phase (they depend on no routing and have the widest entries).
+struct ItemPlan {
+  int r1;           // routed gate/up items
+  int t1, t1s, t2;  // tiles per entry: routed gate/up, shared gate/up, down
+  int S;            // shared-expert entries (0: none); routed entries follow them
+};
+
+template <bool kShared>
+__device__ __forceinline__ Item decode_item(int item, const ItemPlan &ip, const Ws &ws) {
   Item it;
-  if (item < items1) {
-    it.down = 0;
-    it.entry = item / t1;
-    it.tile = item - it.entry * t1;
+  it.shared = 0;
+  if constexpr (!kShared) {
+    if (item < ip.r1) {
+      it.down = 0;
+      it.entry = item / ip.t1;
+      it.tile = item - it.entry * ip.t1;
+    } else {
+      const int j = item - ip.r1;
+      it.down = 1;
+      it.entry = j / ip.t2;
+      it.tile = j - it.entry * ip.t2;
+    }
   } else {
-    const int j = item - items1;
-    it.down = 1;
-    it.entry = j / t2;
-    it.tile = j - it.entry * t2;
+    const int s1 = ip.S * ip.t1s;
+    const int g = s1 + ip.r1;
+    const int s2 = ip.S * ip.t2;
+    int j, t;
+    if (item < s1) {
+      it.down = 0; it.shared = 1; j = item; t = ip.t1s;
+    } else if (item < g) {
+      it.down = 0; j = item - s1; t = ip.t1;
+    } else if (item < g + s2) {
+      it.down = 1; it.shared = 1; j = item - g; t = ip.t2;
+    } else {
+      it.down = 1; j = item - g - s2; t = ip.t2;
+    }
+    const int e = j / t;
+    it.tile = j - e * t;
+    it.entry = it.shared ? e : ip.S + e;
   }
   const int4 en = __ldcg(&ws.entries[it.entry]);
   it.expert = en.x;
@@ -122,6 +153,7 @@ __device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit
   atomicOr(&ws.ctrl[kCtrlErr], bit);
 }
 
+template <bool kShared>
 __global__ void __launch_bounds__(kFfnThreads, 1)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
@@ -173,6 +205,14 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     for (int m = 0; m < kTokBoxSizes && (kTokBox << m) <= d.tok_chunk; ++m) {
       tma_prefetch_desc(&maps.xp[m]);
       tma_prefetch_desc(&maps.act[m]);
+      if constexpr (kShared) {
+        tma_prefetch_desc(&maps.xt[m]);
+        tma_prefetch_desc(&maps.act_s[m]);
+      }
+    }
+    if constexpr (kShared) {
+      tma_prefetch_desc(&maps.w_gu_s);
+      tma_prefetch_desc(&maps.w_down_s);
     }
   }
   if (warp == 1) {
@@ -191,10 +231,15 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   if (blockIdx.x == 0 && threadIdx.x == 0) trace_stamp(ws, tr_step, kTrFfnStart);
 #endif
 
-  const int items1 = __ldcg(&ws.ctrl[kCtrlItems1]);
   const int total = __ldcg(&ws.ctrl[kCtrlTotalItems]);
   const int t1 = d.I / kGateRows;
   const int t2 = d.H / kTileRows;
+  ItemPlan ip;
+  ip.r1 = __ldcg(&ws.ctrl[kCtrlItems1]);
+  ip.t1 = t1;
+  ip.t1s = kShared ? d.Is / kGateRows : 0;
+  ip.t2 = t2;
+  ip.S = kShared ? d.S : 0;
   const int nb_cols = d.tok_chunk;  // TMEM columns per accumulator buffer
 
   if (warp == 0) {
@@ -226,14 +271,15 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           pdl_launch_dependents();
           break;
         }
-        const Item it = decode_item(item, items1, t1, t2, ws);
+        const Item it = decode_item<kShared>(item, ip, ws);
         if (it.down) {
           // the entry's activations must be complete: all its gate/up tiles
           const int *done = &ws.entry_done[it.entry];
-          bool ok = ld_acquire(done) >= t1;
+          const int need = (kShared && it.shared) ? ip.t1s : t1;
+          bool ok = ld_acquire(done) >= need;
           if (!ok) {
             const uint64_t t0 = global_timer_ns();
-            while (!(ok = ld_acquire(done) >= t1)) {
+            while (!(ok = ld_acquire(done) >= need)) {
               if (*abort) break;
               if (global_timer_ns() - t0 > kTimeoutNs) {
                 raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
@@ -245,21 +291,32 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           if (!ok) break;
           fence_proxy_async_global();
         }
-        const int nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
-        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
-        const void *amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
         // the item's token rows: one box of the power-of-two height that
         // covers them (rows past the entry are loaded but not multiplied)
         const int box_m = token_box_for(it.n16);
-        const void *bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
-        int row0, row1;
-        if (it.down) {
-          row0 = it.expert * d.H + it.tile * kTileRows;
-          row1 = row0 + kGateRows;
+        int nsub_total, row0, row1;
+        const void *amap;
+        const void *bmap;
+        if (kShared && it.shared) {
+          // the shared expert: its own weights, tokens in batch order
+          nsub_total = it.down ? d.Is / kBlockK : d.H / kBlockK;
+          amap = it.down ? (const void *)&maps.w_down_s : (const void *)&maps.w_gu_s;
+          bmap = it.down ? (const void *)&maps.act_s[box_m] : (const void *)&maps.xt[box_m];
+          row0 = it.down ? it.tile * kTileRows : it.tile * kGateRows;
+          row1 = it.down ? row0 + kGateRows : row0 + d.Is;
         } else {
-          row0 = it.expert * 2 * d.I + it.tile * kGateRows;
-          row1 = row0 + d.I;
+          nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
+          amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
+          bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
+          if (it.down) {
+            row0 = it.expert * d.H + it.tile * kTileRows;
+            row1 = row0 + kGateRows;
+          } else {
+            row0 = it.expert * 2 * d.I + it.tile * kGateRows;
+            row1 = row0 + d.I;
+          }
         }
+        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         const uint32_t sub_bytes = (uint32_t)(kATileBytes + (kTokBox << box_m) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
@@ -316,7 +373,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           rphase ^= 1u;
         }
         if (item >= total) break;
-        const Item it = decode_item(item, items1, t1, t2, ws);
+        const Item it = decode_item<kShared>(item, ip, ws);
         const int b = local & 1;
         const uint32_t use = (uint32_t)(local >> 1);
         if (!mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, kTimeoutNs)) {
@@ -326,7 +383,8 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(b * nb_cols);
         const uint32_t idesc = idesc_bf16_f32(kTileRows, it.n16 * kTokBox);
-        const int nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
+        const int inner = (kShared && it.shared) ? d.Is : d.I;
+        const int nsub_total = it.down ? inner / kBlockK : d.H / kBlockK;
         const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
@@ -398,7 +456,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
       if (item >= total) break;
       const int b = local & 1;
       if (b != g) continue;
-      const Item it = decode_item(item, items1, t1, t2, ws);
+      const Item it = decode_item<kShared>(item, ip, ws);
       const uint32_t use = (uint32_t)(local >> 1);
       if (!mbar_wait_bounded(accf_bar(b), use & 1u, abort, kTimeoutNs)) {
         if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
@@ -433,8 +491,11 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
               __nv_bfloat162 h2 = __floats2bfloat162_rn(a2[0], a2[1]);
               packed[ii / 2] = *reinterpret_cast<uint32_t *>(&h2);
             }
-            *reinterpret_cast<uint4 *>(ws.act + (size_t)(it.slot_base + col) * d.I +
-                                       it.tile * kGateRows + i0) =
+            // routed: grouped order [B*k, I]; shared: token order [B, Is]
+            __nv_bfloat16 *arow = (kShared && it.shared)
+                                      ? ws.act_s + (size_t)(it.slot_base + col) * d.Is
+                                      : ws.act + (size_t)(it.slot_base + col) * d.I;
+            *reinterpret_cast<uint4 *>(arow + it.tile * kGateRows + i0) =
                 make_uint4(packed[0], packed[1], packed[2], packed[3]);
           }
           epi_bar(g);  // the exchange buffer is rewritten by the next chunk
@@ -448,6 +509,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         if (et == 0) atomicAdd(&ws.entry_done[it.entry], 1);
       } else {
         const int h = it.tile * kTileRows + row;
+        float *ybase = (kShared && it.shared) ? ws.y_s : ws.y;  // token / grouped order
         for (int c = 0; c < it.n16; ++c) {
           uint32_t v[16];
           tmem_ld16(taddr + c * 16, v);
@@ -456,7 +518,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           for (int j = 0; j < 16; ++j) {
             const int col = c * 16 + j;
             if (col < it.n)
-              ws.y[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
+              ybase[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
           }
         }
         tc_fence_before();
@@ -464,12 +526,14 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         __threadfence();
         if (et == 0) *comb_n = 0;
         epi_bar(g);
-        // count this contribution for each token; the k-th one combines
+        // count this contribution for each token; the last of its k routed
+        // (and, with a shared expert, one shared) contributions combines
+        const int last = kShared ? d.k : d.k - 1;
         for (int col = et; col < it.n; col += kEpiThreads) {
-          const int s = __ldcg(&ws.perm[it.slot_base + col]);
-          const int t = s / d.k;
+          const int t = (kShared && it.shared) ? it.slot_base + col
+                                               : __ldcg(&ws.perm[it.slot_base + col]) / d.k;
           const int old = atomicAdd(&ws.comb_cnt[(size_t)t * t2 + it.tile], 1);
-          if (old == d.k - 1) comb_list[atomicAdd(comb_n, 1)] = t;
+          if (old == last) comb_list[atomicAdd(comb_n, 1)] = t;
         }
         __threadfence();
         epi_bar(g);
@@ -507,6 +571,16 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
                 acc.w = fmaf(w, v[jj].w, acc.w);
               }
             }
+          }
+          if constexpr (kShared) {
+            // the shared expert's term, after the k routed ones (Sec. 3.3)
+            const float sg = __ldcg(&ws.shared_gate[t]);
+            const float4 vs = __ldcg(reinterpret_cast<const float4 *>(
+                ws.y_s + (size_t)t * d.H + it.tile * kCombineTile + 4 * lane));
+            acc.x = fmaf(sg, vs.x, acc.x);
+            acc.y = fmaf(sg, vs.y, acc.y);
+            acc.z = fmaf(sg, vs.z, acc.z);
+            acc.w = fmaf(sg, vs.w, acc.w);
           }
           const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
           const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
@@ -564,8 +638,8 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - kCoResidentSmem);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
-  err = cudaFuncSetAttribute(expert_ffn_kernel,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kernel = d.Is > 0 ? expert_ffn_kernel<true> : expert_ffn_kernel<false>;
+  err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
   int tmem_cols = 32;
   while (tmem_cols < 2 * d.tok_chunk) tmem_cols <<= 1;
@@ -580,8 +654,7 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, expert_ffn_kernel, maps, d, ws, out, stages,
-                            tmem_cols);
+  return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols);
 }
 
 }  // namespace slimwise

@@ -12,6 +12,10 @@
 //              at most tok_chunk tokens),
 //   xp         hidden rows copied into grouped order, so the FFN kernel can
 //              stream each expert's tokens with plain 2-D TMA boxes.
+// With a shared expert (Sec. 3.3) it also computes each token's sigmoid gate
+// s_t = 1 / (1 + exp(-w_sg . x_t)), the dot product in the canonical order of
+// the router logits, and lists the shared expert's work entries (the batch in
+// token order, in chunks) ahead of the routed ones.
 // Every CTA recomputes the histogram of the whole batch (B*k ids, a few KB
 // from L2) so the rank of a slot inside its expert, its token-order prefix
 // count, is known without a grid-wide barrier; integer counts make the
@@ -47,8 +51,8 @@ __device__ int warp_exclusive_scan(const int *vals, int *outp, int n, int lane) 
 }
 
 __global__ void __launch_bounds__(kGroupThreads)
-    group_gather_kernel(const __nv_bfloat16 *__restrict__ hidden, Dims d, Ws ws,
-                        int do_gather) {
+    group_gather_kernel(const __nv_bfloat16 *__restrict__ hidden,
+                        const float *__restrict__ w_sg, Dims d, Ws ws, int do_gather) {
   __shared__ int cnt_all[kMaxExperts];
   __shared__ int cnt_before[kMaxExperts];
   __shared__ int offs[kMaxExperts + 1];
@@ -129,15 +133,38 @@ __global__ void __launch_bounds__(kGroupThreads)
       }
 #pragma unroll
       for (int u = 0; u < kVec; ++u) {
-        if (i0 + u * blockDim.x < nt * vecs)
+        if (i0 + u * blockDim.x < nt * vecs) {
           for (int j = 0; j < k; ++j)
             reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[tt[u] * k + j] * H)[vv[u]] = v[u];
+          // token-order copy for the shared expert (a stable address to map)
+          if (d.Is > 0) reinterpret_cast<uint4 *>(ws.xt + (size_t)(t0 + tt[u]) * H)[vv[u]] = v[u];
+        }
       }
     }
   }
   const int ht = H / kCombineTile;
   for (int i = tid; i < (t1 - t0) * ht; i += blockDim.x)
     ws.comb_cnt[(size_t)t0 * ht + i] = 0;
+
+  // shared-expert gate of this CTA's tokens: warp w takes token t0 + w; lane
+  // l accumulates elements 128c + 4l + q (c, q ascending) with fused
+  // multiply-adds, then an xor butterfly over the lanes
+  if (d.Is > 0 && warp < t1 - t0) {
+    const __nv_bfloat16 *xr = hidden + (size_t)(t0 + warp) * H;
+    float p = 0.0f;
+    for (int c = 0; c < H / 128; ++c) {
+      const int h = 128 * c + 4 * lane;
+      const uint2 xv = *reinterpret_cast<const uint2 *>(xr + h);
+      const float4 wv = *reinterpret_cast<const float4 *>(w_sg + h);
+      p = fmaf(__uint_as_float(xv.x << 16), wv.x, p);
+      p = fmaf(__uint_as_float(xv.x & 0xFFFF0000u), wv.y, p);
+      p = fmaf(__uint_as_float(xv.y << 16), wv.z, p);
+      p = fmaf(__uint_as_float(xv.y & 0xFFFF0000u), wv.w, p);
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) p = p + __shfl_xor_sync(0xFFFFFFFFu, p, off);
+    if (lane == 0) ws.shared_gate[t0 + warp] = 1.0f / (1.0f + expf(-p));
+  }
 
   if (blockIdx.x != 0) return;
 
@@ -155,24 +182,30 @@ __global__ void __launch_bounds__(kGroupThreads)
   __syncthreads();
   const int U = flag_scan[E];
   const int n_entries = entry_base[E];
+  // entries [0, n_se) are the shared expert's (expert -1, token order), the
+  // routed ones follow
+  const int n_se = d.S;
   for (int e = tid; e < E; e += blockDim.x) {
     if (cnt_before[e]) ws.union_ids[flag_scan[e]] = e;
     if (e >= U) ws.union_ids[e] = -1;
     const int n_e = offs[e + 1] - offs[e];
     for (int c = 0; c < chunk_cnt[e]; ++c) {
       const int base = c * d.tok_chunk;
-      ws.entries[entry_base[e] + c] =
+      ws.entries[n_se + entry_base[e] + c] =
           make_int4(e, offs[e] + base, min(d.tok_chunk, n_e - base), 0);
     }
   }
-  for (int i = tid; i < n_entries; i += blockDim.x) ws.entry_done[i] = 0;
+  for (int sidx = tid; sidx < n_se; sidx += blockDim.x)
+    ws.entries[sidx] = make_int4(-1, sidx * d.tok_chunk, min(d.tok_chunk, B - sidx * d.tok_chunk), 0);
+  for (int i = tid; i < n_se + n_entries; i += blockDim.x) ws.entry_done[i] = 0;
   if (tid == 0) {
     const int t1_items = d.I / kGateRows;
     const int t2_items = d.H / kTileRows;
+    const int t1s_items = d.Is / kGateRows;
     ws.ctrl[kCtrlUnionSize] = U;
-    ws.ctrl[kCtrlNumEntries] = n_entries;
+    ws.ctrl[kCtrlNumEntries] = n_se + n_entries;
     ws.ctrl[kCtrlItems1] = n_entries * t1_items;
-    ws.ctrl[kCtrlTotalItems] = n_entries * (t1_items + t2_items);
+    ws.ctrl[kCtrlTotalItems] = n_se * (t1s_items + t2_items) + n_entries * (t1_items + t2_items);
     ws.ctrl[kCtrlWorkCounter] = 0;
   }
   __syncthreads();
@@ -182,8 +215,8 @@ __global__ void __launch_bounds__(kGroupThreads)
 #endif
 }
 
-cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
-                                bool pdl, bool gather, cudaStream_t stream) {
+cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shared_gate,
+                                Dims d, Ws ws, bool pdl, bool gather, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((d.B + kGroupTokens - 1) / kGroupTokens);
   cfg.blockDim = dim3(kGroupThreads);
@@ -194,7 +227,7 @@ cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, Dims d, Ws ws,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, group_gather_kernel, hidden, d, ws,
+  return cudaLaunchKernelEx(&cfg, group_gather_kernel, hidden, w_shared_gate, d, ws,
                             gather ? 1 : 0);
 }
 

@@ -94,7 +94,7 @@ int check_shape(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
   return SLIMWISE_OK;
 }
 
-Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
+Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret, int32_t Is = 0) {
   Dims d;
   d.B = s->num_tokens;
   d.H = s->hidden;
@@ -103,14 +103,16 @@ Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
   d.k = top_k;
   d.m_ret = m_ret;
   d.tok_chunk = token_chunk_for(d.B, top_k, m_ret);
+  d.Is = Is;
+  d.S = Is > 0 ? (d.B + d.tok_chunk - 1) / d.tok_chunk : 0;
   return d;
 }
 
 int check_workspace(const slimwise_moe_shape *s, int32_t top_k, void *ws,
-                    size_t ws_bytes, WsLayout *L) {
+                    size_t ws_bytes, WsLayout *L, int32_t Is = 0) {
   if (!ws) return SLIMWISE_ERR_INVALID_ARG;
   if (!aligned(ws, 256)) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
-  *L = make_layout(s->num_tokens, s->hidden, s->num_experts, s->inter, top_k);
+  *L = make_layout(s->num_tokens, s->hidden, s->num_experts, s->inter, top_k, Is);
   return ws_bytes >= L->total ? SLIMWISE_OK : SLIMWISE_ERR_WORKSPACE;
 }
 
@@ -138,26 +140,36 @@ int copy_group_outputs(const Ws &w, const Dims &d, cudaStream_t st, int32_t *cou
 // The FFN kernel's tensor maps for one call.  Encoding them costs host time
 // on every call, so the maps of the last call on this thread are kept and
 // reused while the pointers and sizes they describe are unchanged.
+// The shared expert of Sec. 3.3 (inter == 0: none).
+struct SharedExpert {
+  const float *gate;      // fp32 [H]
+  const void *gate_up;    // bf16 [2 Is, H]
+  const void *down;       // bf16 [H, Is]
+  int32_t inter;          // Is
+};
+
 struct MapsKey {
-  const void *w_gu, *w_down, *xp, *act;
-  int E, H, I, tok_chunk;
+  const void *w_gu, *w_down, *xp, *act, *gu_s, *down_s;
+  int E, H, I, Is, B, tok_chunk;
   uint64_t slots;
   int device;
   bool operator==(const MapsKey &o) const {
-    return w_gu == o.w_gu && w_down == o.w_down && xp == o.xp && act == o.act && E == o.E &&
-           H == o.H && I == o.I && tok_chunk == o.tok_chunk && slots == o.slots &&
+    return w_gu == o.w_gu && w_down == o.w_down && xp == o.xp && act == o.act &&
+           gu_s == o.gu_s && down_s == o.down_s && E == o.E && H == o.H && I == o.I &&
+           Is == o.Is && B == o.B && tok_chunk == o.tok_chunk && slots == o.slots &&
            device == o.device;
   }
 };
 
 bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, const Ws &w,
-                  const Dims &d, uint64_t slots) {
+                  const Dims &d, uint64_t slots, const SharedExpert &se) {
   thread_local bool have = false;
   thread_local MapsKey last;
   thread_local FfnMaps cached;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  const MapsKey key = {w_gate_up, w_down, w.xp, w.act, d.E, d.H, d.I, d.tok_chunk, slots, dev};
+  const MapsKey key = {w_gate_up, w_down, w.xp, w.act, se.gate_up, se.down,
+                       d.E, d.H, d.I, d.Is, d.B, d.tok_chunk, slots, dev};
   if (have && key == last) {
     *maps = cached;
     return true;
@@ -173,6 +185,15 @@ bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, cons
     if (encode_map(&m.xp[b], w.xp, slots, d.H, kTokBox << b) ||
         encode_map(&m.act[b], w.act, slots, d.I, kTokBox << b))
       return false;
+  if (d.Is > 0) {
+    if (encode_map(&m.w_gu_s, se.gate_up, 2 * (uint64_t)d.Is, d.H, kGateRows) ||
+        encode_map(&m.w_down_s, se.down, (uint64_t)d.H, d.Is, kGateRows))
+      return false;
+    for (int b = 0; b < kTokBoxSizes && (kTokBox << b) <= d.tok_chunk; ++b)
+      if (encode_map(&m.xt[b], w.xt, (uint64_t)d.B, d.H, kTokBox << b) ||
+          encode_map(&m.act_s[b], w.act_s, (uint64_t)d.B, d.Is, kTokBox << b))
+        return false;
+  }
   cached = m;
   last = key;
   have = true;
@@ -183,23 +204,32 @@ bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, cons
 int decode_impl(const void *hidden, const float *router_w, const int32_t *retained,
                 int32_t n_retained, const void *w_gate_up, const void *w_down,
                 int32_t top_k, void *out, void *stream, const slimwise_moe_shape *shape,
-                void *workspace, size_t workspace_bytes, const slimwise_decode_opts *opts) {
+                void *workspace, size_t workspace_bytes, const slimwise_decode_opts *opts,
+                const SharedExpert *shared = nullptr) {
   const int32_t m_ret = retained ? n_retained : (shape ? shape->num_experts : 0);
   int rc = check_shape(shape, top_k, m_ret);
   if (rc) return rc;
+  const SharedExpert se = shared ? *shared : SharedExpert{nullptr, nullptr, nullptr, 0};
+  if (shared && (se.inter < 64 || se.inter % 64 != 0 || se.inter > 65536))
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
   if (shape->num_tokens == 0) return SLIMWISE_OK;
+  if (shared) {
+    if (!se.gate || !se.gate_up || !se.down) return SLIMWISE_ERR_INVALID_ARG;
+    if (!aligned(se.gate, 16) || !aligned(se.gate_up, 16) || !aligned(se.down, 16))
+      return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  }
   if (!hidden || !router_w || !w_gate_up || !w_down || !out) return SLIMWISE_ERR_INVALID_ARG;
   if (!aligned(hidden, 16) || !aligned(router_w, 16) || !aligned(w_gate_up, 16) ||
       !aligned(w_down, 16) || !aligned(out, 16) || (retained && !aligned(retained, 4)))
     return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
   WsLayout L;
-  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L);
+  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L, se.inter);
   if (rc) return rc;
   DeviceInfo di;
   rc = device_info(&di);
   if (rc) return rc;
 
-  const Dims d = make_dims(shape, top_k, m_ret);
+  const Dims d = make_dims(shape, top_k, m_ret, se.inter);
   const Ws w = make_ws(workspace, L);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const bool pdl = !(opts && opts->disable_pdl);
@@ -208,7 +238,7 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
 
   FfnMaps maps;
   const uint64_t slots = (uint64_t)d.B * d.k;
-  if (!ffn_maps_for(&maps, w_gate_up, w_down, w, d, slots)) return SLIMWISE_ERR_CUDA;
+  if (!ffn_maps_for(&maps, w_gate_up, w_down, w, d, slots, se)) return SLIMWISE_ERR_CUDA;
 
   // While routing runs, warm L2 with the gate/up weights the FFN streams
   // first -- when the batch almost surely selects every retained expert
@@ -224,7 +254,7 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
   if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained,
                         d, w, pf, pdl, st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
-  if (launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), d, w, pdl, true,
+  if (launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), se.gate, d, w, pdl, true,
                           st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   const bool timed = opts && opts->ffn_begin && opts->ffn_end;
@@ -263,6 +293,31 @@ int slimwise_moe_workspace_size(const slimwise_moe_shape *shape, int32_t top_k,
                        shape->inter, top_k)
                .total;
   return SLIMWISE_OK;
+}
+
+int slimwise_moe_shared_workspace_size(const slimwise_moe_shape *shape, int32_t top_k,
+                                       int32_t inter_shared, size_t *bytes) {
+  if (!bytes) return SLIMWISE_ERR_INVALID_ARG;
+  int rc = check_shape(shape, top_k, shape ? shape->num_experts : 0);
+  if (rc) return rc;
+  if (inter_shared < 64 || inter_shared % 64 != 0 || inter_shared > 65536)
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  *bytes = make_layout(shape->num_tokens, shape->hidden, shape->num_experts,
+                       shape->inter, top_k, inter_shared)
+               .total;
+  return SLIMWISE_OK;
+}
+
+int slimwise_moe_decode_shared(const void *hidden, const float *router_w,
+                               const int32_t *retained_idx, int32_t n_retained,
+                               const void *w_gate_up, const void *w_down, int32_t top_k,
+                               const float *w_shared_gate, const void *w_shared_gate_up,
+                               const void *w_shared_down, int32_t inter_shared, void *out,
+                               void *stream, const slimwise_moe_shape *shape,
+                               void *workspace, size_t workspace_bytes) {
+  const SharedExpert se = {w_shared_gate, w_shared_gate_up, w_shared_down, inter_shared};
+  return decode_impl(hidden, router_w, retained_idx, n_retained, w_gate_up, w_down, top_k,
+                     out, stream, shape, workspace, workspace_bytes, nullptr, &se);
 }
 
 int slimwise_moe_decode(const void *hidden, const float *router_w,
@@ -316,7 +371,7 @@ int slimwise_moe_route(const void *hidden, const float *router_w,
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained_idx,
                         d, w, L2Prefetch{}, false, st) != cudaSuccess ||
-      launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), d, w, false, false,
+      launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), nullptr, d, w, false, false,
                           st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   const size_t slots = (size_t)d.B * d.k;
@@ -348,7 +403,7 @@ int slimwise_moe_group(const int32_t *topk_idx, int32_t top_k, void *stream,
   if (cudaMemsetAsync(w.ctrl + kCtrlErr, 0, 4, st) != cudaSuccess ||
       cudaMemcpyAsync(w.topk_idx, topk_idx, slots * 4, cudaMemcpyDeviceToDevice, st) !=
           cudaSuccess ||
-      launch_group_gather(nullptr, d, w, false, false, st) != cudaSuccess)
+      launch_group_gather(nullptr, nullptr, d, w, false, false, st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   return copy_group_outputs(w, d, st, counts, offsets, union_ids, union_size, perm, pos);
 }

@@ -78,6 +78,16 @@ def hidden_states(batch: int, shape: LayerShape, seed: int, device="cpu") -> tor
     return torch.randn((batch, shape.hidden), generator=g, device=device).to(torch.bfloat16)
 
 
+def shared_expert(hidden: int, inter_shared: int, seed: int, device="cpu"):
+    """Shared expert of one layer: (gate row fp32 [H] ~ N(0, 0.05), gate/up bf16
+    [2Is, H] and down bf16 [H, Is] ~ N(0, 0.02))."""
+    one = LayerShape(hidden=hidden, num_experts=1, inter=inter_shared, top_k=1)
+    gu, dn = expert_weights(one, seed, device=device)
+    g = _gen(seed + 17, device)
+    w_sg = (torch.randn((hidden,), generator=g, device=device) * 0.05).to(torch.float32)
+    return w_sg, gu[0].contiguous(), dn[0].contiguous()
+
+
 def retained_set(num_experts: int, n_retained: int, seed: int, shuffle: bool = False) -> torch.Tensor:
     """int32 ids of the m' experts with the largest U[0,1) importance score.
 

@@ -117,3 +117,35 @@ def test_binding_refuses_cpu_tensors(lib):
     with pytest.raises(TypeError):
         binding.slimwise_moe_decode_full(x, torch.zeros(16, 256), torch.zeros(16, 256, 256, dtype=torch.bfloat16),
                                          torch.zeros(16, 256, 128, dtype=torch.bfloat16), 2)
+
+
+def test_shared_expert_entry_points_validate_without_cuda(lib):
+    P = _fake
+    out = ctypes.c_size_t(0)
+    s64 = binding.Shape(64, 2048, 128, 768)
+    # the workspace grows by the shared expert's gate, token-order hidden
+    # rows, activations and outputs
+    n0 = _ws(64, 2048, 128, 768, 8)
+    assert lib.slimwise_moe_shared_workspace_size(ctypes.byref(s64), 8, 1024, ctypes.byref(out)) == 0
+    assert out.value >= n0 + 64 * (4 + 2 * 2048 + 2 * 1024 + 4 * 2048)
+    s = binding.Shape(4, 256, 16, 128)
+    for bad_is in (0, 32, 96, 1 << 17):
+        assert lib.slimwise_moe_shared_workspace_size(ctypes.byref(s), 2, bad_is, ctypes.byref(out)) == 2
+    big = 1 << 30
+
+    def call(gate=P(), gu=P(), dn=P(), Is=128, ws_bytes=big, shape=s):
+        return lib.slimwise_moe_decode_shared(P(), P(), P(), 8, P(), P(), 2, gate, gu, dn, Is, P(),
+                                              None, ctypes.byref(shape), P(), ws_bytes)
+
+    assert call(Is=96) == 2                 # Is not a multiple of 64
+    assert call(gate=None) == 1             # missing shared gate row
+    assert call(dn=None) == 1               # missing shared down weight
+    assert call(gate=P(0x10004)) == 2       # misaligned gate row
+    assert call(ws_bytes=1024) == 3         # workspace too small
+    # the plain layer's workspace is too small once a shared expert is added
+    n_plain = _ws(4, 256, 16, 128, 2)
+    assert call(ws_bytes=n_plain) == 3
+    # B = 0 is a no-op even with null buffers
+    s0 = binding.Shape(0, 256, 16, 128)
+    assert lib.slimwise_moe_decode_shared(None, None, None, 0, None, None, 2, None, None, None, 128,
+                                          None, None, ctypes.byref(s0), None, 0) == 0

@@ -198,6 +198,75 @@ def test_compact_checkpoint_equals_masked_pool(qwen, m_prime):
     assert int(r_c["union_size"][0]) == int(r_m["union_size"][0])
 
 
+class SharedExpert:
+    def __init__(self, layer, inter_shared, seed):
+        H = layer.shape.hidden
+        self.w_sg, self.gu, self.dn = synth.shared_expert(H, inter_shared, seed)
+        self.gu_bits, self.dn_bits = synth.bf16_bits(self.gu), synth.bf16_bits(self.dn)
+        self.d_w_sg, self.d_gu, self.d_dn = self.w_sg.to(DEV), self.gu.to(DEV), self.dn.to(DEV)
+
+
+def _case_shared(layer, se, B, m_prime, seed_x, seed_imp, k=None, sample=None, x=None):
+    shape = layer.shape
+    k = shape.top_k if k is None else k
+    if x is None:
+        x = synth.hidden_states(B, shape, seed_x)
+    retained = None if m_prime is None else synth.retained_set(shape.num_experts, m_prime, seed_imp)
+    out = sw.slimwise_moe_decode_shared(x.to(DEV), layer.d_wr, None if retained is None else retained.to(DEV),
+                                        layer.d_w_gu, layer.d_w_d, k, se.d_w_sg, se.d_gu, se.d_dn)
+    torch.cuda.synchronize()
+    tokens = None
+    if sample is not None and B > sample:
+        tokens = np.sort(np.random.default_rng(seed_x).choice(B, size=sample, replace=False)).astype(np.int32)
+    ref = oracle.moe_decode_shared(synth.bf16_bits(x), layer.wr.numpy(),
+                                   None if retained is None else retained.numpy(), layer.gu_bits,
+                                   layer.d_bits, k, se.w_sg.numpy(), se.gu_bits, se.dn_bits, tokens)
+    got = out.float().cpu().numpy()
+    if tokens is not None:
+        got = got[tokens]
+    return _check_out(got, ref["out"]), out
+
+
+@pytest.fixture(scope="module")
+def tiny_shared(tiny):
+    return SharedExpert(tiny, 128, seed=31)
+
+
+@pytest.fixture(scope="module")
+def qwen36_shared(qwen36):
+    # Sec. 3.3: the distilled decoder's shared expert is twice the original width
+    return SharedExpert(qwen36, 1024, seed=32)
+
+
+@pytest.mark.parametrize("B", [1, 4, 17, 300])
+def test_shared_expert_layer_tiny(tiny, tiny_shared, B):
+    # B = 300 spans two shared-expert work entries of 256 tokens
+    _case_shared(tiny, tiny_shared, B=B, m_prime=8, seed_x=40 + B, seed_imp=2)
+
+
+@pytest.mark.parametrize("B,m_prime", [(64, 128), (256, 64)])
+def test_shared_expert_layer_qwen36(qwen36, qwen36_shared, B, m_prime):
+    _case_shared(qwen36, qwen36_shared, B=B, m_prime=m_prime, seed_x=50 + B, seed_imp=2 + m_prime,
+                 sample=6)
+
+
+def test_shared_expert_closed_gate_is_the_routed_layer(tiny, tiny_shared):
+    # gate logit -1000 for every token: s_t = 0 and the output is exactly the
+    # routed layer's
+    shape = tiny.shape
+    x = synth.hidden_states(24, shape, 61)
+    x[:, -1] = 1.0
+    w_sg = torch.zeros(shape.hidden, dtype=torch.float32)
+    w_sg[-1] = -1000.0
+    retained = synth.retained_set(shape.num_experts, 8, 2).to(DEV)
+    xd = x.to(DEV)
+    with_se = sw.slimwise_moe_decode_shared(xd, tiny.d_wr, retained, tiny.d_w_gu, tiny.d_w_d, 2,
+                                            w_sg.to(DEV), tiny_shared.d_gu, tiny_shared.d_dn)
+    routed = sw.slimwise_moe_decode(xd, tiny.d_wr, retained, tiny.d_w_gu, tiny.d_w_d, 2)
+    torch.cuda.synchronize()
+    assert torch.equal(with_se, routed)
+
+
 @pytest.mark.parametrize("B", [1, 5, 17, 33, 300])
 def test_ragged_batches_and_token_chunks(tiny, B):
     # k = m' = 8: every token selects every retained expert, so each expert
