@@ -52,6 +52,10 @@ WORKLOADS = {
     "qwen36_p25_b64": dict(B=64, m_prime=192, shape="qwen36"),
     "qwen36_p50_b64": dict(B=64, m_prime=128, shape="qwen36"),
     "qwen36_p75_b64": dict(B=64, m_prime=64, shape="qwen36"),
+    # the same with the distilled decoder's shared expert (Sec. 3.3): one
+    # always-on expert of twice the original width (2 x 512) under a sigmoid gate
+    "qwen36_se_p50_b64": dict(B=64, m_prime=128, shape="qwen36", shared=1024),
+    "qwen36_se_p75_b64": dict(B=64, m_prime=64, shape="qwen36", shared=1024),
 }
 N_BATCHES = 8  # distinct hidden batches rotated through the timed steps
 
@@ -172,13 +176,39 @@ def _pci_bus_id(idx):
 
 # ---------------------------------------------------------------- inputs
 class LayerInputs:
-    def __init__(self, shape, seed, device, copies=1):
+    def __init__(self, shape, seed, device, copies=1, shared=0):
         self.shape = shape
         self.copies = []
         for c in range(copies):
             w_gu, w_d = synth.expert_weights(shape, seed + 7919 * c, device=device)
             self.copies.append((w_gu, w_d))
         self.wr = synth.router_weight(shape, seed, device=device)
+        # shared expert (gate row, gate/up, down) or None
+        self.shared = synth.shared_expert(shape.hidden, shared, seed + 101, device=device) if shared else None
+
+    def shared_bytes(self):
+        """bf16 weight bytes of the shared expert (read every step)."""
+        if self.shared is None:
+            return 0
+        return 2 * (self.shared[1].numel() + self.shared[2].numel())
+
+    def workspace(self, sw, B, device):
+        s = self.shape
+        if self.shared is None:
+            return sw.alloc_workspace(B, s.hidden, s.num_experts, s.inter, s.top_k, device)
+        n = sw.slimwise_moe_shared_workspace_size(B, s.hidden, s.num_experts, s.inter, s.top_k,
+                                                  self.shared[1].shape[0] // 2)
+        return torch.empty(n, dtype=torch.uint8, device=device)
+
+    def call(self, sw, x, retained, w_gu, w_d, out, ws_buf, stream, ffn_events=None):
+        """One layer call through the C ABI."""
+        k = self.shape.top_k
+        if self.shared is None:
+            sw.slimwise_moe_decode_ex(x, self.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
+                                      stream=stream, ffn_events=ffn_events)
+        else:
+            sw.slimwise_moe_decode_shared(x, self.wr, retained, w_gu, w_d, k, *self.shared, out=out,
+                                          workspace=ws_buf, stream=stream, ffn_events=ffn_events)
 
     def compacted(self, m_prime, seed_imp=2):
         """The layer as a compact checkpoint of its m' retained experts."""
@@ -186,6 +216,7 @@ class LayerInputs:
         ret = synth.retained_set(self.shape.num_experts, m_prime, seed_imp).to(self.wr.device)
         c = LayerInputs.__new__(LayerInputs)
         c.shape = synth.LayerShape(self.shape.hidden, m_prime, self.shape.inter, self.shape.top_k)
+        c.shared = self.shared
         c.copies = []
         for (w_gu, w_d) in self.copies:
             gu_c, d_c, wr_c, _ = checkpoint.compact_layer(w_gu, w_d, self.wr, ret)
@@ -230,8 +261,7 @@ def run_layer_steps(sw, layer, hidden_batches, retained, k, steps, stream, ws_bu
         w_gu, w_d = layer.copies[copy_for_step(i)]
         x = hidden_batches[i % len(hidden_batches)]
         ev = None if ffn_events is None else ffn_events[i]
-        sw.slimwise_moe_decode_ex(x, layer.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
-                                  stream=stream, ffn_events=ev)
+        layer.call(sw, x, retained, w_gu, w_d, out, ws_buf, stream, ffn_events=ev)
 
 
 def union_sizes(sw, layer, hidden_batches, retained, k):
@@ -249,11 +279,11 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     batches = [synth.hidden_states(B, shape, seed_x + j, device=device) for j in range(N_BATCHES)]
     retained = None if m_prime >= shape.num_experts else synth.retained_set(
         shape.num_experts, m_prime, 2).to(device)
-    ws_buf = sw.alloc_workspace(B, shape.hidden, shape.num_experts, shape.inter, k, device)
+    ws_buf = layer.workspace(sw, B, device)
     out = torch.empty((B, shape.hidden), dtype=torch.bfloat16, device=device)
     us = union_sizes(sw, layer, batches, retained, k)
     u_mean = float(np.mean(us))
-    touched = u_mean * shape.expert_bytes
+    touched = u_mean * shape.expert_bytes + layer.shared_bytes()
     ncopies = len(layer.copies)
     rotate = touched < 4 * L2_BYTES and ncopies > 1
     copy_for_step = (lambda i: i % ncopies) if rotate else (lambda i: 0)
@@ -296,6 +326,8 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
         raise RuntimeError(f"device error bits {flags:#x}")
     ffn_bytes = touched + 2 * B * shape.hidden * 2          # union weights + hidden in + out
     layer_bytes = touched + m_prime * shape.hidden * 4 + 2 * B * shape.hidden * 2
+    if layer.shared is not None:
+        layer_bytes += shape.hidden * 4  # shared-expert gate row
     return {
         "B": B, "m_prime": m_prime, "union_mean": u_mean, "union_eq1": m_prime * (1 - (1 - k / m_prime) ** B),
         "step_ms": step_ms, "tokens_per_s": B / (step_ms * 1e-3),
@@ -355,8 +387,7 @@ def e2e_measure(sw, layer, B, m_prime, steps, device, point):
     def one(i):
         dev_in.copy_(host_in[i % len(host_in)], non_blocking=True)
         w_gu, w_d = layer.copies[copy_for_step(i)]
-        sw.slimwise_moe_decode_ex(dev_in, layer.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
-                                  stream=stream)
+        layer.call(sw, dev_in, retained, w_gu, w_d, out, ws_buf, stream)
         host_out.copy_(out, non_blocking=True)
 
     for i in range(5):
@@ -391,10 +422,16 @@ def cpu_baseline(layer, B, m_prime, budget_s=15.0):
     idx, gates = oracle.route(z, ret, shape.top_k)
     oracle.group_by_expert(idx, shape.num_experts)
     t_route = time.perf_counter() - t0
+    se = None
+    if layer.shared is not None:
+        se = [t.cpu() for t in layer.shared]
+        se = (se[0].numpy(), synth.bf16_bits(se[1]), synth.bf16_bits(se[2]))
     n, t_ffn = 0, 0.0
     while n < B and t_ffn < budget_s:
         t1 = time.perf_counter()
-        oracle.experts_combine(x, idx, gates, gu, dn, tokens=[n])
+        o = oracle.experts_combine(x, idx, gates, gu, dn, tokens=[n])
+        if se is not None:
+            oracle.shared_expert_add(x, se[0], se[1], se[2], o, tokens=[n])
         t_ffn += time.perf_counter() - t1
         n += 1
     per_token = t_ffn / n + t_route / B
@@ -418,8 +455,8 @@ def main_gpu(args, ws, rank, local):
     # one weight copy is enough when the touched bytes exceed L2 several times;
     # the sweep rotates 4 copies for its small-batch points
     copies = 4 if args.sweep else 1
-    layer = LayerInputs(shape, seed=0, device=device, copies=copies)
-    sweep_layer = layer
+    layer = LayerInputs(shape, seed=0, device=device, copies=copies, shared=wl.get("shared", 0))
+    sweep_layer = layer if layer.shared is None else LayerInputs(shape, 0, device, copies)
     if wl.get("compact"):
         layer = layer.compacted(m_prime)
         shape = layer.shape
@@ -444,10 +481,11 @@ def main_gpu(args, ws, rank, local):
         "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
                    "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B,
                    "form": "compact checkpoint" if wl.get("compact") else "masked pool",
+                   "shared_expert_inter": wl.get("shared", 0),
                    "union_mean": pt["union_mean"], "union_eq1": pt["union_eq1"],
                    "parallelism": f"replicas{ws}",
                    "l2": "touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
-                         % (pt["union_mean"] * shape.expert_bytes / 1e9)},
+                         % ((pt["union_mean"] * shape.expert_bytes + layer.shared_bytes()) / 1e9)},
         "touched_hbm": {"gbs": pt["touched_gbs"], "frac_of_8tbs": pt["touched_gbs"] / NOMINAL_HBM_GBS,
                         "frac_of_measured": pt["touched_gbs"] / peak},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -553,6 +591,10 @@ def main_reference(args, ws, rank):
     wr = synth.router_weight(shape, 0).numpy()
     gu, dn = synth.bf16_bits(w_gu), synth.bf16_bits(w_d)
     ret = None if m_prime >= shape.num_experts else synth.retained_set(shape.num_experts, m_prime, 2).numpy()
+    se = None
+    if wl.get("shared"):
+        w_sg, gu_s, dn_s = synth.shared_expert(shape.hidden, wl["shared"], 0 + 101)
+        se = (w_sg.numpy(), synth.bf16_bits(gu_s), synth.bf16_bits(dn_s))
     if wl.get("compact"):
         # the retained experts' rows only, in ascending id order
         ids = np.sort(ret)
@@ -570,7 +612,9 @@ def main_reference(args, ws, rank):
         t_route = time.perf_counter() - t0
         toks = [(i * sample + j) % B for j in range(sample)]
         t1 = time.perf_counter()
-        oracle.experts_combine(x, idx, gates, gu, dn, tokens=toks)
+        o = oracle.experts_combine(x, idx, gates, gu, dn, tokens=toks)
+        if se is not None:
+            oracle.shared_expert_add(x, se[0], se[1], se[2], o, tokens=toks)
         t_ffn = time.perf_counter() - t1
         return t_route / B + t_ffn / sample   # seconds per token
 

@@ -207,6 +207,18 @@ int slimwise_moe_decode_shared(const void *hidden, const float *router_w,
                                const slimwise_moe_shape *shape, void *workspace,
                                size_t workspace_bytes);
 
+/* slimwise_moe_decode_shared with the launch options of slimwise_moe_decode_ex. */
+int slimwise_moe_decode_shared_ex(const void *hidden, const float *router_w,
+                                  const int32_t *retained_idx, int32_t n_retained,
+                                  const void *w_gate_up, const void *w_down,
+                                  int32_t top_k, const float *w_shared_gate,
+                                  const void *w_shared_gate_up,
+                                  const void *w_shared_down, int32_t inter_shared,
+                                  void *out, void *stream,
+                                  const slimwise_moe_shape *shape, void *workspace,
+                                  size_t workspace_bytes,
+                                  const slimwise_decode_opts *opts);
+
 /*
  * slimwise_moe_decode for callers that cannot allocate device memory (an
  * engine that reserved all of its memory up front, a plugin handed only its

@@ -33,6 +33,7 @@ EXPORTED = (
     "slimwise_moe_decode_full", "slimwise_moe_decode_ex", "slimwise_moe_route",
     "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
     "slimwise_moe_shared_workspace_size", "slimwise_moe_decode_shared",
+    "slimwise_moe_decode_shared_ex",
 )
 
 
@@ -81,6 +82,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
             lib.slimwise_moe_shared_workspace_size.argtypes = [SP, i32, i32, ctypes.POINTER(sz)]
             lib.slimwise_moe_decode_shared.argtypes = [P, P, P, i32, P, P, i32, P, P, P, i32,
                                                        P, P, SP, P, sz]
+            lib.slimwise_moe_decode_shared_ex.argtypes = [P, P, P, i32, P, P, i32, P, P, P, i32,
+                                                          P, P, SP, P, sz,
+                                                          ctypes.POINTER(DecodeOpts)]
             for name in EXPORTED[1:]:
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
@@ -159,9 +163,11 @@ def slimwise_moe_shared_workspace_size(num_tokens: int, hidden: int, num_experts
 
 def slimwise_moe_decode_shared(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
                                w_shared_gate, w_shared_gate_up, w_shared_down, out=None,
-                               workspace=None, stream=None):
+                               workspace=None, stream=None, ffn_events=None, disable_pdl=False,
+                               grid_ctas=0):
     """Decode MoE layer with a shared expert under a sigmoid gate (Sec. 3.3);
-    retained_idx None = full pool.  Returns `out`."""
+    retained_idx None = full pool.  Launch options as slimwise_moe_decode_ex.
+    Returns `out`."""
     _dev(hidden, torch.bfloat16, "hidden")
     _dev(router_w, torch.float32, "router_w")
     _dev(w_gate_up, torch.bfloat16, "w_gate_up")
@@ -182,11 +188,16 @@ def slimwise_moe_decode_shared(hidden, router_w, retained_idx, w_gate_up, w_down
     if retained_idx is not None:
         _dev(retained_idx, torch.int32, "retained_idx")
         n_ret = int(retained_idx.numel())
-    _check(load().slimwise_moe_decode_shared(
-        _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),
-        int(top_k), _ptr(w_shared_gate), _ptr(w_shared_gate_up), _ptr(w_shared_down),
-        inter_shared, _ptr(out), _stream(stream), ctypes.byref(s), _ptr(workspace),
-        workspace.numel()), "slimwise_moe_decode_shared")
+    args = (_ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),
+            int(top_k), _ptr(w_shared_gate), _ptr(w_shared_gate_up), _ptr(w_shared_down),
+            inter_shared, _ptr(out), _stream(stream), ctypes.byref(s), _ptr(workspace),
+            workspace.numel())
+    if ffn_events is None and not disable_pdl and not grid_ctas:
+        _check(load().slimwise_moe_decode_shared(*args), "slimwise_moe_decode_shared")
+    else:
+        opts = _opts(ffn_events, disable_pdl, grid_ctas)
+        _check(load().slimwise_moe_decode_shared_ex(*args, ctypes.byref(opts)),
+               "slimwise_moe_decode_shared_ex")
     return out
 
 
@@ -213,6 +224,14 @@ def slimwise_moe_decode_full(hidden, router_w, w_gate_up, w_down, top_k, out=Non
     return out
 
 
+def _opts(ffn_events, disable_pdl, grid_ctas):
+    opts = DecodeOpts(None, None, int(bool(disable_pdl)), int(grid_ctas))
+    if ffn_events is not None:
+        opts.ffn_begin = ctypes.c_void_p(ffn_events[0].cuda_event)
+        opts.ffn_end = ctypes.c_void_p(ffn_events[1].cuda_event)
+    return opts
+
+
 def slimwise_moe_decode_ex(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
                            out=None, workspace=None, stream=None, ffn_events=None,
                            disable_pdl=False, grid_ctas=0):
@@ -224,10 +243,7 @@ def slimwise_moe_decode_ex(hidden, router_w, retained_idx, w_gate_up, w_down, to
     s, out, workspace = _prep(hidden, router_w, w_gate_up, w_down, top_k, out, workspace)
     if retained_idx is not None:
         _dev(retained_idx, torch.int32, "retained_idx")
-    opts = DecodeOpts(None, None, int(bool(disable_pdl)), int(grid_ctas))
-    if ffn_events is not None:
-        opts.ffn_begin = ctypes.c_void_p(ffn_events[0].cuda_event)
-        opts.ffn_end = ctypes.c_void_p(ffn_events[1].cuda_event)
+    opts = _opts(ffn_events, disable_pdl, grid_ctas)
     n_ret = 0 if retained_idx is None else int(retained_idx.numel())
     _check(load().slimwise_moe_decode_ex(
         _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),

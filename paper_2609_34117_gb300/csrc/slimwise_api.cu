@@ -320,6 +320,19 @@ int slimwise_moe_decode_shared(const void *hidden, const float *router_w,
                      out, stream, shape, workspace, workspace_bytes, nullptr, &se);
 }
 
+int slimwise_moe_decode_shared_ex(const void *hidden, const float *router_w,
+                                  const int32_t *retained_idx, int32_t n_retained,
+                                  const void *w_gate_up, const void *w_down, int32_t top_k,
+                                  const float *w_shared_gate, const void *w_shared_gate_up,
+                                  const void *w_shared_down, int32_t inter_shared, void *out,
+                                  void *stream, const slimwise_moe_shape *shape,
+                                  void *workspace, size_t workspace_bytes,
+                                  const slimwise_decode_opts *opts) {
+  const SharedExpert se = {w_shared_gate, w_shared_gate_up, w_shared_down, inter_shared};
+  return decode_impl(hidden, router_w, retained_idx, n_retained, w_gate_up, w_down, top_k,
+                     out, stream, shape, workspace, workspace_bytes, opts, &se);
+}
+
 int slimwise_moe_decode(const void *hidden, const float *router_w,
                         const int32_t *retained_idx, int32_t n_retained,
                         const void *w_gate_up, const void *w_down, int32_t top_k,
