@@ -60,6 +60,10 @@ def _load():
             lib.oracle_experts_combine.restype = i32
             lib.oracle_shared_expert_add.argtypes = [P, P, P, P, i32, i32, P, i32, P, P]
             lib.oracle_shared_expert_add.restype = i32
+            lib.oracle_expert_stats.argtypes = [P, P, P, P, i32, i32, i32, i32, i32, P]
+            lib.oracle_expert_stats.restype = i32
+            lib.oracle_select_retained.argtypes = [P, i32, i32, i32, P]
+            lib.oracle_select_retained.restype = i32
             lib.oracle_moe_decode.argtypes = [P, P, P, i32, P, P, i32, i32, i32, i32, i32, P, P, P]
             lib.oracle_moe_decode.restype = i32
             _lib = lib
@@ -180,6 +184,40 @@ def shared_expert_add(x_bf16, w_shared_gate, w_shared_gu, w_shared_down, out, to
     return s
 
 
+CRITERIA = {"mass": 0, "ean": 1, "reap": 2}
+
+
+def expert_stats(x_bf16, router_w, w_gate_up, w_down, k, stats=None):
+    """Sec. 2.3 importance statistics of one calibration batch, full pool:
+    fp64 [E, 4] = (tokens routed, routing mass, EAN, REAP numerator), added
+    to `stats` when given."""
+    x = _c(x_bf16, np.uint16)
+    w = _c(router_w, np.float32)
+    wgu = _c(w_gate_up, np.uint16)
+    wd = _c(w_down, np.uint16)
+    B, H = x.shape
+    E = w.shape[0]
+    I = wgu.shape[1] // 2
+    if stats is None:
+        stats = np.zeros((E, 4), np.float64)
+    assert stats.dtype == np.float64 and stats.shape == (E, 4) and stats.flags.c_contiguous
+    rc = _load().oracle_expert_stats(_ptr(x), _ptr(w), _ptr(wgu), _ptr(wd), B, H, E, I, k, _ptr(stats))
+    if rc != 0:
+        raise ValueError("oracle_expert_stats")
+    return stats
+
+
+def select_retained(stats, m_prime, criterion):
+    """Top-m' experts by `criterion` ('mass', 'ean' or 'reap'), ties to the
+    lowest id; int32 ids ascending."""
+    st = _c(stats, np.float64)
+    E = st.shape[0]
+    ids = np.empty(m_prime, np.int32)
+    if _load().oracle_select_retained(_ptr(st), E, int(m_prime), CRITERIA[criterion], _ptr(ids)) != 0:
+        raise ValueError("oracle_select_retained: bad arguments")
+    return ids
+
+
 def moe_decode(x_bf16, router_w, retained, w_gate_up, w_down, k):
     """Whole decode layer over the retained pool (retained=None: full pool).
 
@@ -262,7 +300,7 @@ class swapped_library:
         lib = ctypes.CDLL(self.path)
         for name in ("oracle_router_logits", "oracle_route", "oracle_group_by_expert",
                      "oracle_expert_swiglu", "oracle_experts_combine", "oracle_moe_decode",
-                     "oracle_shared_expert_add"):
+                     "oracle_shared_expert_add", "oracle_expert_stats", "oracle_select_retained"):
             fn_new, fn_old = getattr(lib, name), getattr(base, name)
             fn_new.argtypes, fn_new.restype = fn_old.argtypes, fn_old.restype
         with _lock:

@@ -301,3 +301,86 @@ int oracle_moe_decode(const uint16_t *x, const float *router_w,
   free(z); free(tokens);
   return rc;
 }
+
+/*
+ * Expert-importance statistics over calibration tokens (Sec. 2.3: routing
+ * mass aggregates gate probabilities, EAN measures expert output norms, REAP
+ * weights those norms by the gates; App. A: one pass over the calibration
+ * data with the full pool).  Routing over the full pool as in
+ * oracle_moe_decode; for each token t and each of its k selections e with
+ * gate g and expert output y = y^{(e)}(x_t), tokens in order:
+ *   stats[e*4 + 0] += 1                 tokens routed to e
+ *   stats[e*4 + 1] += g                 routing mass
+ *   stats[e*4 + 2] += ||y||_2           expert activation norm (EAN)
+ *   stats[e*4 + 3] += g * ||y||_2       REAP numerator (score: / count)
+ * stats: fp64 [E, 4], accumulated into.  Returns 0, or -1 on failure.
+ */
+int oracle_expert_stats(const uint16_t *x, const float *router_w,
+                        const uint16_t *w_gate_up, const uint16_t *w_down,
+                        int B, int H, int E, int I, int k, double *stats) {
+  if (B == 0) return 0;
+  float *z = (float *)malloc(sizeof(float) * (size_t)B * E);
+  int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * (size_t)B * k);
+  double *gates = (double *)malloc(sizeof(double) * (size_t)B * k);
+  double *a = (double *)malloc(sizeof(double) * (size_t)I);
+  double *y = (double *)malloc(sizeof(double) * (size_t)H);
+  int rc = -1;
+  if (z && idx && gates && a && y) {
+    oracle_router_logits(x, router_w, B, H, E, z);
+    rc = oracle_route(z, B, E, NULL, 0, k, idx, gates);
+    for (int t = 0; rc == 0 && t < B; ++t)
+      for (int j = 0; j < k; ++j) {
+        const int e = idx[(size_t)t * k + j];
+        const double g = gates[(size_t)t * k + j];
+        oracle_expert_swiglu(x + (size_t)t * H, w_gate_up + (size_t)e * 2 * I * H,
+                             w_down + (size_t)e * H * I, H, I, a, y);
+        double n2 = 0.0;
+        for (int h = 0; h < H; ++h) n2 += y[h] * y[h];
+        const double nrm = sqrt(n2);
+        stats[(size_t)e * 4 + 0] += 1.0;
+        stats[(size_t)e * 4 + 1] += g;
+        stats[(size_t)e * 4 + 2] += nrm;
+        stats[(size_t)e * 4 + 3] += g * nrm;
+      }
+  }
+  free(z); free(idx); free(gates); free(a); free(y);
+  return rc;
+}
+
+/*
+ * Retained set K' from the statistics (Sec. 3.1: rank the layer's experts by
+ * an importance criterion and keep the top m').  Score of expert e:
+ *   criterion 0  routing mass   stats[e*4 + 1]
+ *   criterion 1  EAN            stats[e*4 + 2]
+ *   criterion 2  REAP           stats[e*4 + 3] / stats[e*4 + 0]  (0 if unrouted)
+ * The m' highest scores are kept, ties to the lowest id; ids ascending.
+ * Returns 0, or -1 on bad arguments.
+ */
+int oracle_select_retained(const double *stats, int E, int m_prime,
+                           int criterion, int32_t *ids) {
+  if (m_prime < 0 || m_prime > E || criterion < 0 || criterion > 2) return -1;
+  double *score = (double *)malloc(sizeof(double) * (size_t)(E > 0 ? E : 1));
+  char *taken = (char *)calloc((size_t)(E > 0 ? E : 1), 1);
+  if (!score || !taken) {
+    free(score); free(taken);
+    return -1;
+  }
+  for (int e = 0; e < E; ++e) {
+    const double *st = stats + (size_t)e * 4;
+    if (criterion == 0) score[e] = st[1];
+    else if (criterion == 1) score[e] = st[2];
+    else score[e] = st[0] > 0.0 ? st[3] / st[0] : 0.0;
+  }
+  /* m' rounds of arg-max over the remaining experts */
+  for (int r = 0; r < m_prime; ++r) {
+    int best = -1;
+    for (int e = 0; e < E; ++e)
+      if (!taken[e] && (best < 0 || score[e] > score[best])) best = e;
+    taken[best] = 1;
+  }
+  int n = 0;
+  for (int e = 0; e < E; ++e)
+    if (taken[e]) ids[n++] = e;
+  free(score); free(taken);
+  return 0;
+}

@@ -33,6 +33,13 @@ MUTATIONS = {
     "shared_gate_sign": ("double s = 1.0 / (1.0 + exp(-(double)z));", "double s = 1.0 / (1.0 + exp((double)z));"),
     # shared expert: gate not applied
     "shared_gate_dropped": ("for (int h = 0; h < H; ++h) o[h] += s * y[h];", "for (int h = 0; h < H; ++h) o[h] += y[h];"),
+    # statistics: activation norm squared instead of the norm
+    "stats_norm_squared": ("stats[(size_t)e * 4 + 2] += nrm;", "stats[(size_t)e * 4 + 2] += n2;"),
+    # statistics: REAP without the gate
+    "stats_reap_no_gate": ("stats[(size_t)e * 4 + 3] += g * nrm;", "stats[(size_t)e * 4 + 3] += nrm;"),
+    # selection: ties to the highest id
+    "select_tie_highest": ("if (!taken[e] && (best < 0 || score[e] > score[best])) best = e;",
+                           "if (!taken[e] && (best < 0 || score[e] >= score[best])) best = e;"),
     # grouping: offsets off by one expert
     "offsets_shift": ("offsets[e + 1] = offsets[e] + counts[e];", "offsets[e + 1] = offsets[e] + counts[e > 0 ? e - 1 : 0];"),
     # grouping: token order reversed inside an expert
@@ -53,6 +60,8 @@ PIN_FUNCS = [
     (pins.test_shared_expert_gate_is_sigmoid_of_canonical_logit, ()),
     (pins.test_shared_expert_saturated_gates, ()),
     (pins.test_shared_expert_twice_width_is_sum_of_halves, ()),
+    (pins.test_expert_stats_totals_and_one_hot_router, ()),
+    (pins.test_select_retained_matches_brute_force_with_ties, (0,)),
 ]
 
 

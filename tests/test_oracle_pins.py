@@ -376,3 +376,66 @@ def test_shared_expert_twice_width_is_sum_of_halves(oracle_lib):
     dn_init = np.concatenate([dn1, np.zeros_like(dn2)], axis=1)
     init, _ = _shared_only(oracle_lib, xb, w_sg, gu, dn_init)
     assert np.array_equal(init, a)
+
+
+# --------------------------------------------------------------------------
+# Expert-importance statistics and the retained set (Sec. 2.3, Sec. 3.1)
+# --------------------------------------------------------------------------
+def test_expert_stats_totals_and_one_hot_router(oracle_lib):
+    # every token makes k selections whose gates sum to one
+    shape = synth.TINY
+    x, wr, w_gu, w_d = _tiny_layer(B=12)
+    xb, w, gu, dn = _bits(x), wr.numpy(), _bits(w_gu), _bits(w_d)
+    st = oracle_lib.expert_stats(xb, w, gu, dn, 2)
+    assert st[:, 0].sum() == 12 * 2
+    assert abs(st[:, 1].sum() - 12.0) < 1e-12
+    assert np.all(st >= 0) and np.all(st[st[:, 0] == 0] == 0)
+    # statistics accumulate over calibration batches
+    st2 = oracle_lib.expert_stats(xb, w, gu, dn, 2, stats=st.copy())
+    np.testing.assert_allclose(st2, 2 * st, rtol=1e-15, atol=0)
+    # top-1 one-hot router: every token goes to e* with gate 1, so EAN is the
+    # sum of the dense SwiGLU output norms and REAP is EAN / count
+    e_star = 5
+    x1, wr1 = synth.apply_popularity_bias(x, wr, torch.zeros(shape.num_experts))
+    wr1[e_star, -1] = 8.0
+    xb1, w1 = _bits(x1), wr1.numpy()
+    st1 = oracle_lib.expert_stats(xb1, w1, gu, dn, 1)
+    x64 = _bf16_to_f64(xb1)
+    norms = [np.linalg.norm(_dense_swiglu(x64[t], _bf16_to_f64(gu[e_star]), _bf16_to_f64(dn[e_star])))
+             for t in range(12)]
+    assert st1[e_star, 0] == 12 and st1[e_star, 1] == 12.0
+    np.testing.assert_allclose(st1[e_star, 2], sum(norms), rtol=1e-11)
+    np.testing.assert_allclose(st1[e_star, 3], sum(norms), rtol=1e-11)
+    assert np.all(np.delete(st1, e_star, axis=0) == 0)
+    ids = oracle_lib.select_retained(st1, 1, "reap")
+    assert list(ids) == [e_star]
+    # zero router: every token selects experts 0..k-1 with gate exactly 1/k,
+    # so each REAP numerator is its EAN / k and each mass is count / k
+    k = 4
+    st0 = oracle_lib.expert_stats(xb, np.zeros_like(w), gu, dn, k)
+    assert np.all(st0[:k, 0] == 12) and np.all(st0[k:] == 0)
+    np.testing.assert_allclose(st0[:k, 1], 12 / k, rtol=1e-14)
+    np.testing.assert_allclose(st0[:k, 3], st0[:k, 2] / k, rtol=1e-13)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_select_retained_matches_brute_force_with_ties(oracle_lib, seed):
+    rng = np.random.default_rng(seed)
+    E = 24
+    st = np.zeros((E, 4))
+    st[:, 0] = rng.integers(0, 4, E)
+    # few distinct values: many ties
+    st[:, 1] = rng.integers(0, 3, E) * 0.5
+    st[:, 2] = rng.integers(0, 3, E) * 0.25
+    st[:, 3] = st[:, 2] * st[:, 1]
+    for crit in ("mass", "ean", "reap"):
+        if crit == "mass":
+            score = st[:, 1]
+        elif crit == "ean":
+            score = st[:, 2]
+        else:
+            score = np.where(st[:, 0] > 0, st[:, 3] / np.maximum(st[:, 0], 1), 0.0)
+        for m in (0, 1, 7, E):
+            # brute force: sort by (score desc, id asc), keep m, report ascending
+            order = sorted(range(E), key=lambda e: (-score[e], e))[:m]
+            assert list(oracle_lib.select_retained(st, m, crit)) == sorted(order)
