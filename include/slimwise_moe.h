@@ -220,6 +220,42 @@ int slimwise_moe_decode_shared_ex(const void *hidden, const float *router_w,
                                   const slimwise_decode_opts *opts);
 
 /*
+ * Expert-importance statistics of one calibration batch (Sec. 2.3: routing
+ * mass, Expert Activation Norm, REAP; collected with the full pool, App. A).
+ * Runs the full-pool layer (its output goes to `out`, bf16 [B, H]) and, for
+ * each expert e and each token t that selected it, with gate g and expert
+ * output y (before gating), adds to the caller's fp64 [E, 4] device buffer:
+ *   stats[e][0] += 1,  stats[e][1] += g,  stats[e][2] += ||y||_2,
+ *   stats[e][3] += g * ||y||_2
+ * Tokens are taken in order for each expert.  The buffer is caller-owned and
+ * accumulates across calls (zero it before the first batch).  Other
+ * arguments as slimwise_moe_decode_full; stats must be 8-byte aligned.
+ */
+int slimwise_moe_expert_stats(const void *hidden, const float *router_w,
+                              const void *w_gate_up, const void *w_down,
+                              int32_t top_k, double *stats, void *out,
+                              void *stream, const slimwise_moe_shape *shape,
+                              void *workspace, size_t workspace_bytes);
+
+enum {
+  SLIMWISE_CRITERION_MASS = 0, /* score = routing mass stats[e][1]               */
+  SLIMWISE_CRITERION_EAN = 1,  /* score = activation norm sum stats[e][2]        */
+  SLIMWISE_CRITERION_REAP = 2  /* score = stats[e][3] / stats[e][0] (0 unrouted) */
+};
+
+/*
+ * Retained set K' from the statistics (Sec. 3.1: rank the layer's experts by
+ * an importance criterion, keep the top m'): the n_retained experts of
+ * highest score, ties to the lowest id, written ascending to retained_idx
+ * (device int32 [n_retained]) -- ready for slimwise_moe_decode or for building
+ * the compact checkpoint.  stats: device fp64 [num_experts, 4].  One kernel
+ * launch on `stream`; num_experts <= 1024.
+ */
+int slimwise_moe_select_retained(const double *stats, int32_t num_experts,
+                                 int32_t n_retained, int32_t criterion,
+                                 int32_t *retained_idx, void *stream);
+
+/*
  * slimwise_moe_decode for callers that cannot allocate device memory (an
  * engine that reserved all of its memory up front, a plugin handed only its
  * inputs and outputs): the same layer, with the scratch memory taken from a

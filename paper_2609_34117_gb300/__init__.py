@@ -14,8 +14,10 @@ from .binding import (  # noqa: F401
     slimwise_moe_decode_full,
     slimwise_moe_decode_shared,
     slimwise_moe_device_status,
+    slimwise_moe_expert_stats,
     slimwise_moe_group,
     slimwise_moe_route,
+    slimwise_moe_select_retained,
     slimwise_moe_shared_workspace_size,
     slimwise_moe_workspace_size,
 )

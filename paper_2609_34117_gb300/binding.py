@@ -33,7 +33,7 @@ EXPORTED = (
     "slimwise_moe_decode_full", "slimwise_moe_decode_ex", "slimwise_moe_route",
     "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
     "slimwise_moe_shared_workspace_size", "slimwise_moe_decode_shared",
-    "slimwise_moe_decode_shared_ex",
+    "slimwise_moe_decode_shared_ex", "slimwise_moe_expert_stats", "slimwise_moe_select_retained",
 )
 
 
@@ -85,6 +85,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
             lib.slimwise_moe_decode_shared_ex.argtypes = [P, P, P, i32, P, P, i32, P, P, P, i32,
                                                           P, P, SP, P, sz,
                                                           ctypes.POINTER(DecodeOpts)]
+            lib.slimwise_moe_expert_stats.argtypes = [P, P, P, P, i32, P, P, P, SP, P, sz]
+            lib.slimwise_moe_select_retained.argtypes = [P, i32, i32, i32, P, P]
             for name in EXPORTED[1:]:
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
@@ -222,6 +224,34 @@ def slimwise_moe_decode_full(hidden, router_w, w_gate_up, w_down, top_k, out=Non
         _stream(stream), ctypes.byref(s), _ptr(workspace), workspace.numel()),
         "slimwise_moe_decode_full")
     return out
+
+
+CRITERIA = {"mass": 0, "ean": 1, "reap": 2}
+
+
+def slimwise_moe_expert_stats(hidden, router_w, w_gate_up, w_down, top_k, stats=None, out=None,
+                              workspace=None, stream=None):
+    """One calibration batch of importance statistics (Sec. 2.3), full pool.
+    `stats` (fp64 [E, 4], device) accumulates; returns (stats, layer output)."""
+    s, out, workspace = _prep(hidden, router_w, w_gate_up, w_down, top_k, out, workspace)
+    if stats is None:
+        stats = torch.zeros((s.num_experts, 4), dtype=torch.float64, device=hidden.device)
+    _dev(stats, torch.float64, "stats")
+    _check(load().slimwise_moe_expert_stats(
+        _ptr(hidden), _ptr(router_w), _ptr(w_gate_up), _ptr(w_down), int(top_k), _ptr(stats),
+        _ptr(out), _stream(stream), ctypes.byref(s), _ptr(workspace), workspace.numel()),
+        "slimwise_moe_expert_stats")
+    return stats, out
+
+
+def slimwise_moe_select_retained(stats, n_retained, criterion="reap", stream=None):
+    """Retained set from statistics: int32 [n_retained] device ids, ascending."""
+    _dev(stats, torch.float64, "stats")
+    ids = torch.empty(int(n_retained), dtype=torch.int32, device=stats.device)
+    _check(load().slimwise_moe_select_retained(_ptr(stats), int(stats.shape[0]), int(n_retained),
+                                               CRITERIA[criterion], _ptr(ids), _stream(stream)),
+           "slimwise_moe_select_retained")
+    return ids
 
 
 def _opts(ffn_events, disable_pdl, grid_ctas):

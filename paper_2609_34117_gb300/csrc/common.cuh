@@ -219,6 +219,12 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
                               __nv_bfloat16 *out, int grid, bool pdl,
                               cudaStream_t stream);
 
+// Importance statistics of the last full-pool call in `ws` added to stats
+// (fp64 [E, 4]); retained set from statistics (criterion 0 mass, 1 EAN, 2 REAP).
+cudaError_t launch_expert_stats(Dims d, Ws ws, double *stats, cudaStream_t stream);
+cudaError_t launch_select_retained(const double *stats, int E, int m_prime, int criterion,
+                                   int32_t *ids, cudaStream_t stream);
+
 #if defined(__CUDACC__)
 // ---------------------------------------------------------------------------
 // Device helpers

@@ -333,6 +333,45 @@ int slimwise_moe_decode_shared_ex(const void *hidden, const float *router_w,
                      out, stream, shape, workspace, workspace_bytes, opts, &se);
 }
 
+int slimwise_moe_expert_stats(const void *hidden, const float *router_w,
+                              const void *w_gate_up, const void *w_down, int32_t top_k,
+                              double *stats, void *out, void *stream,
+                              const slimwise_moe_shape *shape, void *workspace,
+                              size_t workspace_bytes) {
+  int rc = check_shape(shape, top_k, shape ? shape->num_experts : 0);
+  if (rc) return rc;
+  if (shape->num_tokens == 0) return SLIMWISE_OK;
+  if (!stats) return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(stats, 8)) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  // the full-pool layer (its output is the calibration pass's layer output)
+  rc = decode_impl(hidden, router_w, nullptr, 0, w_gate_up, w_down, top_k, out, stream, shape,
+                   workspace, workspace_bytes, nullptr);
+  if (rc) return rc;
+  WsLayout L;
+  rc = check_workspace(shape, top_k, workspace, workspace_bytes, &L);
+  if (rc) return rc;
+  const Dims d = make_dims(shape, top_k, shape->num_experts);
+  return launch_expert_stats(d, make_ws(workspace, L), stats,
+                             reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? SLIMWISE_OK
+             : SLIMWISE_ERR_CUDA;
+}
+
+int slimwise_moe_select_retained(const double *stats, int32_t num_experts, int32_t n_retained,
+                                 int32_t criterion, int32_t *retained_idx, void *stream) {
+  if (num_experts < 1 || num_experts > kMaxExperts) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  if (n_retained < 0 || n_retained > num_experts) return SLIMWISE_ERR_INVALID_ARG;
+  if (criterion < SLIMWISE_CRITERION_MASS || criterion > SLIMWISE_CRITERION_REAP)
+    return SLIMWISE_ERR_INVALID_ARG;
+  if (n_retained == 0) return SLIMWISE_OK;
+  if (!stats || !retained_idx) return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(stats, 8) || !aligned(retained_idx, 4)) return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  return launch_select_retained(stats, num_experts, n_retained, criterion, retained_idx,
+                                reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? SLIMWISE_OK
+             : SLIMWISE_ERR_CUDA;
+}
+
 int slimwise_moe_decode(const void *hidden, const float *router_w,
                         const int32_t *retained_idx, int32_t n_retained,
                         const void *w_gate_up, const void *w_down, int32_t top_k,

@@ -149,3 +149,23 @@ def test_shared_expert_entry_points_validate_without_cuda(lib):
     s0 = binding.Shape(0, 256, 16, 128)
     assert lib.slimwise_moe_decode_shared(None, None, None, 0, None, None, 2, None, None, None, 128,
                                           None, None, ctypes.byref(s0), None, 0) == 0
+
+
+def test_statistics_entry_points_validate_without_cuda(lib):
+    P = _fake
+    s = binding.Shape(4, 256, 16, 128)
+    big = 1 << 30
+    # null statistics buffer; misaligned one
+    assert lib.slimwise_moe_expert_stats(P(), P(), P(), P(), 2, None, P(), None, ctypes.byref(s), P(), big) == 1
+    assert lib.slimwise_moe_expert_stats(P(), P(), P(), P(), 2, P(0x10004), P(), None, ctypes.byref(s), P(), big) == 2
+    # bad shape is reported before anything else
+    bad = binding.Shape(4, 100, 16, 128)
+    assert lib.slimwise_moe_expert_stats(P(), P(), P(), P(), 2, P(), P(), None, ctypes.byref(bad), P(), big) == 2
+    s0 = binding.Shape(0, 256, 16, 128)
+    assert lib.slimwise_moe_expert_stats(None, None, None, None, 2, None, None, None, ctypes.byref(s0), None, 0) == 0
+    # selection: pool too large, m' out of range, unknown criterion, null outputs
+    assert lib.slimwise_moe_select_retained(P(), 2000, 8, 2, P(), None) == 2
+    assert lib.slimwise_moe_select_retained(P(), 16, 17, 2, P(), None) == 1
+    assert lib.slimwise_moe_select_retained(P(), 16, 8, 3, P(), None) == 1
+    assert lib.slimwise_moe_select_retained(None, 16, 8, 2, P(), None) == 1
+    assert lib.slimwise_moe_select_retained(P(), 16, 0, 2, None, None) == 0

@@ -396,3 +396,53 @@ def test_zipf_skewed_layers_route_exactly(qwen):
         r = sw.slimwise_moe_route(x.to(DEV), wr.to(DEV), ret.to(DEV), 8, shape.num_experts, shape.inter)
         us.append(int(r["union_size"].item()))
     assert np.mean(us) < m_prime * (1 - (1 - 8 / m_prime) ** Bs)
+
+
+# --------------------------------------------------------------------------
+# Expert-importance statistics and the retained set (Sec. 2.3, Sec. 3.1)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("layer_name,B,k", [("tiny", 40, 2), ("qwen", 64, 8)])
+def test_expert_stats_match_oracle(request, layer_name, B, k):
+    layer = request.getfixturevalue(layer_name)
+    shape = layer.shape
+    stats = None
+    ref = np.zeros((shape.num_experts, 4))
+    for batch in range(2):   # statistics accumulate over calibration batches
+        x = synth.hidden_states(B, shape, 70 + batch)
+        stats, out = sw.slimwise_moe_expert_stats(x.to(DEV), layer.d_wr, layer.d_w_gu, layer.d_w_d, k,
+                                                  stats=stats)
+        ref = oracle.expert_stats(synth.bf16_bits(x), layer.wr.numpy(), layer.gu_bits, layer.d_bits, k,
+                                  stats=ref)
+        # the calibration pass's layer output is the full-pool layer
+        full = sw.slimwise_moe_decode_full(x.to(DEV), layer.d_wr, layer.d_w_gu, layer.d_w_d, k)
+        torch.cuda.synchronize()
+        assert torch.equal(out, full)
+    got = stats.cpu().numpy()
+    assert np.array_equal(got[:, 0], ref[:, 0])                      # tokens routed: exact
+    np.testing.assert_allclose(got[:, 1], ref[:, 1], rtol=1e-5, atol=1e-6)   # fp32 gates
+    # norms of fp32 expert outputs computed through a bf16 activation
+    np.testing.assert_allclose(got[:, 2], ref[:, 2], rtol=1e-2, atol=1e-6)
+    np.testing.assert_allclose(got[:, 3], ref[:, 3], rtol=1e-2, atol=1e-6)
+    # the device selection is the oracle's selection of the same statistics
+    for crit in ("mass", "ean", "reap"):
+        for m in (1, shape.num_experts // 2, shape.num_experts):
+            ids = sw.slimwise_moe_select_retained(stats, m, crit).cpu().numpy()
+            assert np.array_equal(ids, oracle.select_retained(got, m, crit)), (crit, m)
+
+
+def test_select_retained_ties_and_extremes():
+    E = 100
+    rng = np.random.default_rng(5)
+    st = np.zeros((E, 4))
+    st[:, 0] = rng.integers(0, 3, E)
+    st[:, 1] = rng.integers(0, 4, E) * 0.25
+    st[:, 2] = rng.integers(0, 4, E) * 0.5
+    st[:, 3] = st[:, 1] * st[:, 2]
+    d = torch.from_numpy(st).to(DEV)
+    for crit in ("mass", "ean", "reap"):
+        for m in (0, 1, 37, E):
+            ids = sw.slimwise_moe_select_retained(d, m, crit).cpu().numpy()
+            assert np.array_equal(ids, oracle.select_retained(st, m, crit)), (crit, m)
+    # all scores equal: the lowest ids
+    z = torch.zeros((E, 4), dtype=torch.float64, device=DEV)
+    assert np.array_equal(sw.slimwise_moe_select_retained(z, 10, "reap").cpu().numpy(), np.arange(10))
