@@ -26,7 +26,7 @@
 namespace {
 
 // Scratch limit: enough for the Qwen-class layer (H = 2048, E = 128,
-// I = 768, top-8) at decode batches up to 128 tokens.
+// I = 768, top-8) at decode batches up to 151 tokens.
 constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
