@@ -185,20 +185,9 @@ struct Dims {
 };
 
 // Kernel launch declarations (defined in their own translation units).
-// L2 warm-up issued by the routing kernel while HBM would otherwise idle: the
-// gate/up weights of the first `n_experts` retained experts (in the order of
-// the retained list), which the expert FFN streams first when they are in the
-// batch's union.  A prefetch only moves data into L2; results do not depend on it.
-struct L2Prefetch {
-  const char *base;      // w_gate_up
-  size_t expert_stride;  // bytes from one expert's gate/up block to the next
-  size_t bytes;          // bytes of each expert to prefetch
-  int n_experts;         // 0: no prefetch
-};
-
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
-                              const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
-                              bool pdl, cudaStream_t stream);
+                              const int32_t *retained, Dims d, Ws ws, bool pdl,
+                              cudaStream_t stream);
 // w_shared_gate: fp32 [H] gate row of the shared expert, or NULL (d.Is == 0).
 cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shared_gate,
                                 Dims d, Ws ws, bool pdl, bool gather, cudaStream_t stream);
@@ -340,6 +329,9 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map,
       "tx::bytes.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar), "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");

@@ -84,14 +84,29 @@ struct StageType<4> {
 // Shared memory of one CTA: hidden rows [TB][H] (StageType), logits of its
 // slice [TB][slice] fp32, retained ids [m] int32.  Rows of tokens past the
 // batch are zero, so every token slot computes (and discards) a logit.
-template <int TB>
+// Round j of the top-k: the winner (order bits whi, complemented id wlo) goes
+// to lane j.  With no candidate left (fewer than k distinct ids, already
+// reported) a valid id stands in.
+__device__ __forceinline__ void take_winner(uint32_t whi, uint32_t wlo, int j, int lane,
+                                            const int32_t *ids, const Dims &d, float &my_z,
+                                            int &my_e) {
+  uint32_t wid = 0xFFFFFFFFu - wlo;
+  if (whi == 0u || wid >= (uint32_t)d.E) wid = (uint32_t)ids[0];
+  if (lane == j) {
+    my_z = logit_from_order_bits(whi);
+    my_e = (int)wid;
+  }
+}
+
+// TB tokens per cluster; NC candidates per lane in the register top-k
+// (m' <= 32 NC), or NC = 0 for the general top-k of larger pools.
+template <int TB, int NC>
 // Two CTAs per SM worth of registers: a routing CTA must fit beside a
 // persistent expert-FFN CTA so it can be resident before that grid ends.
 __global__ void __launch_bounds__(kRouteThreads, 2)
     route_topk_kernel(const __nv_bfloat16 *__restrict__ hidden,
                       const float *__restrict__ router_w,
-                      const int32_t *__restrict__ retained, Dims d, Ws ws,
-                      L2Prefetch pf) {
+                      const int32_t *__restrict__ retained, Dims d, Ws ws) {
   using XT = typename StageType<TB>::T;
   extern __shared__ __align__(16) unsigned char smem[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -102,6 +117,20 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * sizeof(XT));
   int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)TB * slice);
 
+  // Before waiting for the previous kernel on the stream (this CTA may be
+  // resident while it finishes): warm L2 with this CTA's router rows.  These
+  // are prefetches only -- no value read here is used, and the ids that
+  // address them are read past L1 -- so the results do not depend on whether
+  // the previous kernel wrote the router rows or the retained ids.
+  {
+    const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
+    const int lpr = H / 32;  // 128-byte lines per fp32 router row
+    for (int i = threadIdx.x; i < (r_hi - r_lo) * lpr; i += blockDim.x) {
+      const int r = r_lo + i / lpr;
+      const int e = min(max(retained ? __ldcg(retained + r) : r, 0), d.E - 1);
+      prefetch_l2(router_w + (size_t)e * H + (size_t)(i % lpr) * 32);
+    }
+  }
   // The inputs may come from the previous kernel on the stream.
   pdl_wait_primary();
   // Let the grouping kernel become resident; it waits for this grid to end.
@@ -165,20 +194,6 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   }
   __syncthreads();
 
-  // L2 warm-up: 64 KiB pieces of the first pf.n_experts experts' gate/up
-  // weights, spread over all CTAs of the grid.
-  if (threadIdx.x == 0 && pf.n_experts > 0) {
-    constexpr uint32_t kPiece = 65536;
-    const size_t per_expert = (pf.bytes + kPiece - 1) / kPiece;
-    const size_t pieces = per_expert * (size_t)min(pf.n_experts, m);
-    for (size_t p = blockIdx.x; p < pieces; p += gridDim.x) {
-      const size_t e_i = p / per_expert, off = (p - e_i * per_expert) * kPiece;
-      const uint32_t len = (uint32_t)min((size_t)kPiece, pf.bytes - off);
-      const char *src = pf.base + (size_t)ids[e_i] * pf.expert_stride + off;
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(len) : "memory");
-    }
-  }
-
   // Logits of this CTA's slice [r_lo, r_hi) of the retained list.
   const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
   const int nchunks = H / 128;
@@ -210,55 +225,90 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   // Top-k and gates: warp w of CTA 0 handles token w of the cluster.
   if (crank == 0 && warp < nt) {
     const int t = t0 + warp;
-    // this lane's candidates r = lane + 32 i as 64-bit keys (order-preserving
-    // logit bits, complemented id), sorted descending; the remote loads of
-    // four candidates are issued before any is used
-    unsigned long long key[kMaxExperts / 32];
-    int nc = 0;
-    for (int r0 = lane; r0 < m; r0 += 128) {
-      float zc[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int r = r0 + 32 * u;
-        if (r < m) {
-          const int owner = r / slice;
-          zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int r = r0 + 32 * u;
-        if (r < m) {
-          const unsigned long long kv = ((unsigned long long)logit_order_bits(zc[u]) << 32) |
-                                        (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r]);
-          int i = nc++;
-          while (i > 0 && key[i - 1] < kv) {
-            key[i] = key[i - 1];
-            --i;
-          }
-          key[i] = kv;
-        }
-      }
-    }
-    // k rounds: the warp's largest head key wins and its lane pops it
-    int head = 0;
     float my_z = 0.0f;
     int my_e = 0;
-    for (int j = 0; j < k; ++j) {
-      const unsigned long long mine = head < nc ? key[head] : 0ull;
-      const uint32_t hi = (uint32_t)(mine >> 32), lo = (uint32_t)mine;
-      const uint32_t whi = __reduce_max_sync(0xFFFFFFFFu, hi);
-      const uint32_t wlo = __reduce_max_sync(0xFFFFFFFFu, hi == whi ? lo : 0u);
-      const unsigned long long win = ((unsigned long long)whi << 32) | wlo;
-      // pop every copy of the winner (repeated retained ids give equal keys)
-      while (head < nc && key[head] == win) ++head;
-      uint32_t wid = 0xFFFFFFFFu - wlo;
-      // no candidate left (fewer than k distinct ids, already reported):
-      // fall back to a valid id
-      if (whi == 0u || wid >= (uint32_t)d.E) wid = (uint32_t)ids[0];
-      if (lane == j) {
-        my_z = logit_from_order_bits(whi);
-        my_e = (int)wid;
+    if constexpr (NC > 0) {
+      // this lane's candidates r = lane + 32 i (i < NC) as 64-bit keys
+      // (order-preserving logit bits, complemented id; 0 = none), kept sorted
+      // descending in registers -- every index below is a compile-time one;
+      // all remote loads are issued before any is used
+      float zc[NC];
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        const int r = lane + 32 * i;
+        if (r < m) {
+          const int owner = r / slice;
+          zc[i] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
+        }
+      }
+      unsigned long long key[NC];
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        const int r = lane + 32 * i;
+        key[i] = r < m ? ((unsigned long long)logit_order_bits(zc[i]) << 32) |
+                             (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r])
+                       : 0ull;
+#pragma unroll
+        for (int j = i; j > 0; --j)
+          if (key[j] > key[j - 1]) {
+            const unsigned long long tmp = key[j];
+            key[j] = key[j - 1];
+            key[j - 1] = tmp;
+          }
+      }
+      // k rounds: the warp's largest head key wins and its lane pops it
+      for (int j = 0; j < k; ++j) {
+        const unsigned long long mine = key[0];
+        const uint32_t hi = (uint32_t)(mine >> 32), lo = (uint32_t)mine;
+        const uint32_t whi = __reduce_max_sync(0xFFFFFFFFu, hi);
+        const uint32_t wlo = __reduce_max_sync(0xFFFFFFFFu, hi == whi ? lo : 0u);
+        const unsigned long long win = ((unsigned long long)whi << 32) | wlo;
+        // pop every copy of the winner (repeated retained ids give equal keys)
+        for (int pops = 0; pops < NC && key[0] == win && win != 0ull; ++pops) {
+#pragma unroll
+          for (int i = 0; i + 1 < NC; ++i) key[i] = key[i + 1];
+          key[NC - 1] = 0ull;
+        }
+        take_winner(whi, wlo, j, lane, ids, d, my_z, my_e);
+      }
+    } else {
+      // large pools: the lane's candidates sorted in a local array
+      unsigned long long key[kMaxExperts / 32];
+      int nc = 0;
+      for (int r0 = lane; r0 < m; r0 += 128) {
+        float zc[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int r = r0 + 32 * u;
+          if (r < m) {
+            const int owner = r / slice;
+            zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int r = r0 + 32 * u;
+          if (r < m) {
+            const unsigned long long kv = ((unsigned long long)logit_order_bits(zc[u]) << 32) |
+                                          (unsigned long long)(0xFFFFFFFFu - (uint32_t)ids[r]);
+            int i = nc++;
+            while (i > 0 && key[i - 1] < kv) {
+              key[i] = key[i - 1];
+              --i;
+            }
+            key[i] = kv;
+          }
+        }
+      }
+      int head = 0;
+      for (int j = 0; j < k; ++j) {
+        const unsigned long long mine = head < nc ? key[head] : 0ull;
+        const uint32_t hi = (uint32_t)(mine >> 32), lo = (uint32_t)mine;
+        const uint32_t whi = __reduce_max_sync(0xFFFFFFFFu, hi);
+        const uint32_t wlo = __reduce_max_sync(0xFFFFFFFFu, hi == whi ? lo : 0u);
+        const unsigned long long win = ((unsigned long long)whi << 32) | wlo;
+        while (head < nc && key[head] == win) ++head;
+        take_winner(whi, wlo, j, lane, ids, d, my_z, my_e);
       }
     }
     // g_j = exp(z_j - z_1) / sum_j' exp(z_j' - z_1), the sum in j order.
@@ -280,15 +330,15 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
 #endif
 }
 
-template <int TB>
+template <int TB, int NC>
 cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
-                            const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
-                            bool pdl, cudaStream_t stream) {
+                            const int32_t *retained, Dims d, Ws ws, bool pdl,
+                            cudaStream_t stream) {
   const int slice = (d.m_ret + kClusterCtas - 1) / kClusterCtas;
   const size_t smem = (size_t)TB * d.H * sizeof(typename StageType<TB>::T) +
                       (size_t)TB * slice * 4 + (size_t)d.m_ret * 4;
   cudaError_t err = cudaFuncSetAttribute(
-      route_topk_kernel<TB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      route_topk_kernel<TB, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(((d.B + TB - 1) / TB) * kClusterCtas);
@@ -304,16 +354,25 @@ cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, route_topk_kernel<TB>, hidden, router_w, retained, d, ws, pf);
+  return cudaLaunchKernelEx(&cfg, route_topk_kernel<TB, NC>, hidden, router_w, retained, d, ws);
+}
+
+template <int TB>
+cudaError_t launch_route_nc(const __nv_bfloat16 *hidden, const float *router_w,
+                            const int32_t *retained, Dims d, Ws ws, bool pdl,
+                            cudaStream_t stream) {
+  if (d.m_ret <= 128) return launch_route_tb<TB, 4>(hidden, router_w, retained, d, ws, pdl, stream);
+  if (d.m_ret <= 256) return launch_route_tb<TB, 8>(hidden, router_w, retained, d, ws, pdl, stream);
+  return launch_route_tb<TB, 0>(hidden, router_w, retained, d, ws, pdl, stream);
 }
 
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
-                              const int32_t *retained, Dims d, Ws ws, L2Prefetch pf,
-                              bool pdl, cudaStream_t stream) {
-  if (d.B <= 32) return launch_route_tb<1>(hidden, router_w, retained, d, ws, pf, pdl, stream);
-  if (d.B <= 64) return launch_route_tb<2>(hidden, router_w, retained, d, ws, pf, pdl, stream);
-  if (d.B <= 256) return launch_route_tb<4>(hidden, router_w, retained, d, ws, pf, pdl, stream);
-  return launch_route_tb<8>(hidden, router_w, retained, d, ws, pf, pdl, stream);
+                              const int32_t *retained, Dims d, Ws ws, bool pdl,
+                              cudaStream_t stream) {
+  if (d.B <= 32) return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
+  if (d.B <= 64) return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
+  if (d.B <= 256) return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);
+  return launch_route_nc<8>(hidden, router_w, retained, d, ws, pdl, stream);
 }
 
 }  // namespace slimwise

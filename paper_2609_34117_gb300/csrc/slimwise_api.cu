@@ -12,14 +12,7 @@
 
 using namespace slimwise;
 
-// Retained experts whose gate/up weights the routing kernel prefetches into L2.
-#ifndef SLIMWISE_L2_PREFETCH_EXPERTS
-#define SLIMWISE_L2_PREFETCH_EXPERTS 0
-#endif
-
 namespace {
-
-constexpr int kL2PrefetchExperts = SLIMWISE_L2_PREFETCH_EXPERTS;
 
 struct DeviceInfo {
   int sms = 0;
@@ -240,19 +233,8 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
   const uint64_t slots = (uint64_t)d.B * d.k;
   if (!ffn_maps_for(&maps, w_gate_up, w_down, w, d, slots, se)) return SLIMWISE_ERR_CUDA;
 
-  // While routing runs, warm L2 with the gate/up weights the FFN streams
-  // first -- when the batch almost surely selects every retained expert
-  // (Eq. 1: 1 - (1 - k/m')^B close to 1).
-  L2Prefetch pf = {};
-  const double cover = 1.0 - std::pow(1.0 - (double)top_k / m_ret, (double)d.B);
-  if (kL2PrefetchExperts > 0 && cover >= 0.9) {
-    pf.base = static_cast<const char *>(w_gate_up);
-    pf.expert_stride = (size_t)2 * d.I * d.H * 2;
-    pf.bytes = pf.expert_stride;
-    pf.n_experts = std::min(m_ret, kL2PrefetchExperts);
-  }
   if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained,
-                        d, w, pf, pdl, st) != cudaSuccess)
+                        d, w, pdl, st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   if (launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), se.gate, d, w, pdl, true,
                           st) != cudaSuccess)
@@ -422,7 +404,7 @@ int slimwise_moe_route(const void *hidden, const float *router_w,
   const Ws w = make_ws(workspace, L);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (launch_route_topk(static_cast<const __nv_bfloat16 *>(hidden), router_w, retained_idx,
-                        d, w, L2Prefetch{}, false, st) != cudaSuccess ||
+                        d, w, false, st) != cudaSuccess ||
       launch_group_gather(static_cast<const __nv_bfloat16 *>(hidden), nullptr, d, w, false, false,
                           st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
