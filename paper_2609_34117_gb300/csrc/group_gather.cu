@@ -55,6 +55,7 @@ __global__ void __launch_bounds__(kGroupThreads)
                         const float *__restrict__ w_sg, Dims d, Ws ws, int do_gather) {
   __shared__ int cnt_all[kMaxExperts];
   __shared__ int cnt_before[kMaxExperts];
+  __shared__ int union_flag[kMaxExperts];
   __shared__ int offs[kMaxExperts + 1];
   __shared__ int flag_scan[kMaxExperts + 1];
   __shared__ int chunk_cnt[kMaxExperts];
@@ -76,7 +77,23 @@ __global__ void __launch_bounds__(kGroupThreads)
   const int S = B * k;
   const int t0 = blockIdx.x * kGroupTokens;
   const int t1 = min(B, t0 + kGroupTokens);
+  const int nt = t1 - t0;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int vecs = H / 8;  // 16-byte vectors per hidden row
+
+  // This CTA's hidden rows go into registers first, so that their loads
+  // overlap the histogram below (up to kPre vectors per thread).
+  constexpr int kPre = 4;
+  const bool early = do_gather && nt * vecs <= kPre * (int)blockDim.x;
+  uint4 hv[kPre];
+  if (early) {
+#pragma unroll
+    for (int u = 0; u < kPre; ++u) {
+      const int i = tid + u * blockDim.x;
+      if (i < nt * vecs)
+        hv[u] = __ldg(reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + i / vecs) * H) + i % vecs);
+    }
+  }
 
   for (int e = tid; e < E; e += blockDim.x) {
     cnt_all[e] = 0;
@@ -84,7 +101,7 @@ __global__ void __launch_bounds__(kGroupThreads)
   }
   if (tid == 0) bad = 0;
   __syncthreads();
-  const int nslots = (t1 - t0) * k;
+  const int nslots = nt * k;
   for (int s = tid; s < S; s += blockDim.x) {
     int e = ws.topk_idx[s];
     if (e < 0 || e >= E) {  // only possible for caller-given selections
@@ -96,7 +113,16 @@ __global__ void __launch_bounds__(kGroupThreads)
     else if (s < t1 * k) my_ids[s - t0 * k] = e;
   }
   __syncthreads();
+  // offsets of the experts; union flags and work-entry counts (every CTA has
+  // the whole histogram, so each can publish its share of the results)
+  for (int e = tid; e < E; e += blockDim.x) {
+    union_flag[e] = cnt_all[e] > 0 ? 1 : 0;
+    chunk_cnt[e] = (cnt_all[e] + d.tok_chunk - 1) / d.tok_chunk;
+  }
+  __syncthreads();
   if (warp == 0) warp_exclusive_scan(cnt_all, offs, E, lane);
+  if (warp == 1) warp_exclusive_scan(union_flag, flag_scan, E, lane);
+  if (warp == 2) warp_exclusive_scan(chunk_cnt, entry_base, E, lane);
   __syncthreads();
 
   // Grouped position of each of this CTA's slots: offset of the expert plus
@@ -114,11 +140,21 @@ __global__ void __launch_bounds__(kGroupThreads)
     ws.pos[s] = p;
     ws.perm[p] = s;
   }
-  if (do_gather) {
-    // each token row is loaded once into registers and stored to its k
-    // grouped positions; four vectors per thread in flight
-    const int vecs = H / 8;  // 16-byte vectors per row
-    const int nt = t1 - t0;
+  if (early) {
+    // each token row, already in registers, goes to its k grouped positions
+#pragma unroll
+    for (int u = 0; u < kPre; ++u) {
+      const int i = tid + u * blockDim.x;
+      if (i < nt * vecs) {
+        const int tt = i / vecs, vv = i % vecs;
+        for (int j = 0; j < k; ++j)
+          reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[tt * k + j] * H)[vv] = hv[u];
+        // token-order copy for the shared expert (a stable address to map)
+        if (d.Is > 0) reinterpret_cast<uint4 *>(ws.xt + (size_t)(t0 + tt) * H)[vv] = hv[u];
+      }
+    }
+  } else if (do_gather) {
+    // wide rows: loaded here, four vectors per thread in flight
     constexpr int kVec = 4;
     for (int i0 = tid; i0 < nt * vecs; i0 += kVec * blockDim.x) {
       uint4 v[kVec];
@@ -136,20 +172,19 @@ __global__ void __launch_bounds__(kGroupThreads)
         if (i0 + u * blockDim.x < nt * vecs) {
           for (int j = 0; j < k; ++j)
             reinterpret_cast<uint4 *>(ws.xp + (size_t)my_pos[tt[u] * k + j] * H)[vv[u]] = v[u];
-          // token-order copy for the shared expert (a stable address to map)
           if (d.Is > 0) reinterpret_cast<uint4 *>(ws.xt + (size_t)(t0 + tt[u]) * H)[vv[u]] = v[u];
         }
       }
     }
   }
   const int ht = H / kCombineTile;
-  for (int i = tid; i < (t1 - t0) * ht; i += blockDim.x)
+  for (int i = tid; i < nt * ht; i += blockDim.x)
     ws.comb_cnt[(size_t)t0 * ht + i] = 0;
 
   // shared-expert gate of this CTA's tokens: warp w takes token t0 + w; lane
   // l accumulates elements 128c + 4l + q (c, q ascending) with fused
   // multiply-adds, then an xor butterfly over the lanes
-  if (d.Is > 0 && warp < t1 - t0) {
+  if (d.Is > 0 && warp < nt) {
     const __nv_bfloat16 *xr = hidden + (size_t)(t0 + warp) * H;
     float p = 0.0f;
     for (int c = 0; c < H / 128; ++c) {
@@ -166,27 +201,17 @@ __global__ void __launch_bounds__(kGroupThreads)
     if (lane == 0) ws.shared_gate[t0 + warp] = 1.0f / (1.0f + expf(-p));
   }
 
-  if (blockIdx.x != 0) return;
-
-  // CTA 0 publishes the batch-wide results and the FFN work list.
-  for (int e = tid; e < E; e += blockDim.x) {
-    ws.counts[e] = cnt_all[e];
-    ws.offsets[e] = offs[e];
-    cnt_before[e] = cnt_all[e] > 0 ? 1 : 0;  // reuse as union flags
-    chunk_cnt[e] = (cnt_all[e] + d.tok_chunk - 1) / d.tok_chunk;
-  }
-  if (tid == 0) ws.offsets[E] = offs[E];
-  __syncthreads();
-  if (warp == 0) warp_exclusive_scan(cnt_before, flag_scan, E, lane);
-  if (warp == 1) warp_exclusive_scan(chunk_cnt, entry_base, E, lane);
-  __syncthreads();
+  // The batch-wide results and the FFN work list, each expert written by one
+  // thread of the grid.  Entries [0, n_se) are the shared expert's (expert
+  // -1, token order); the routed ones follow.
   const int U = flag_scan[E];
   const int n_entries = entry_base[E];
-  // entries [0, n_se) are the shared expert's (expert -1, token order), the
-  // routed ones follow
   const int n_se = d.S;
-  for (int e = tid; e < E; e += blockDim.x) {
-    if (cnt_before[e]) ws.union_ids[flag_scan[e]] = e;
+  const int gtid = blockIdx.x * blockDim.x + tid, gstride = gridDim.x * blockDim.x;
+  for (int e = gtid; e < E; e += gstride) {
+    ws.counts[e] = cnt_all[e];
+    ws.offsets[e] = offs[e];
+    if (union_flag[e]) ws.union_ids[flag_scan[e]] = e;
     if (e >= U) ws.union_ids[e] = -1;
     const int n_e = offs[e + 1] - offs[e];
     for (int c = 0; c < chunk_cnt[e]; ++c) {
@@ -195,13 +220,14 @@ __global__ void __launch_bounds__(kGroupThreads)
           make_int4(e, offs[e] + base, min(d.tok_chunk, n_e - base), 0);
     }
   }
-  for (int sidx = tid; sidx < n_se; sidx += blockDim.x)
+  for (int sidx = gtid; sidx < n_se; sidx += gstride)
     ws.entries[sidx] = make_int4(-1, sidx * d.tok_chunk, min(d.tok_chunk, B - sidx * d.tok_chunk), 0);
-  for (int i = tid; i < n_se + n_entries; i += blockDim.x) ws.entry_done[i] = 0;
-  if (tid == 0) {
+  for (int i = gtid; i < n_se + n_entries; i += gstride) ws.entry_done[i] = 0;
+  if (blockIdx.x == 0 && tid == 0) {
     const int t1_items = d.I / kGateRows;
     const int t2_items = d.H / kTileRows;
     const int t1s_items = d.Is / kGateRows;
+    ws.offsets[E] = offs[E];
     ws.ctrl[kCtrlUnionSize] = U;
     ws.ctrl[kCtrlNumEntries] = n_se + n_entries;
     ws.ctrl[kCtrlItems1] = n_entries * t1_items;
@@ -209,9 +235,9 @@ __global__ void __launch_bounds__(kGroupThreads)
     ws.ctrl[kCtrlWorkCounter] = 0;
   }
   __syncthreads();
-  if (tid == 0 && bad) atomicOr(&ws.ctrl[kCtrlErr], bad);
+  if (blockIdx.x == 0 && tid == 0 && bad) atomicOr(&ws.ctrl[kCtrlErr], bad);
 #ifdef SLIMWISE_TRACE
-  if (tid == 0) trace_stamp(ws, tr_step, kTrGroupEnd);
+  if (blockIdx.x == 0 && tid == 0) trace_stamp(ws, tr_step, kTrGroupEnd);
 #endif
 }
 
