@@ -89,6 +89,15 @@ __host__ __device__ inline size_t align_up(size_t v, size_t a) {
   return (v + a - 1) / a * a;
 }
 
+// Work entries the workspace has room for: one per selected expert plus one
+// per further chunk (the chunk size depends on m', so bounded by the smallest
+// chunk), plus the shared expert's chunks of the batch.
+__host__ __device__ inline int max_entries_for(int B, int E, int k, int Is) {
+  const long long slots = (long long)B * k;
+  return E + (int)((slots + kMinTokChunk - 1) / kMinTokChunk) +
+         (Is > 0 ? (B + kMinTokChunk - 1) / kMinTokChunk : 0);
+}
+
 // Is: intermediate width of the shared expert (0: none).
 inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
   WsLayout L;
@@ -99,11 +108,7 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
     o = align_up(o + (bytes ? bytes : 1), 1024);
     return r;
   };
-  // entries: one per selected expert plus one per further chunk; the chunk
-  // size depends on m', so bound it by the smallest chunk; the shared expert
-  // adds one entry per chunk of the batch
-  L.max_entries = E + (int32_t)((slots + kMinTokChunk - 1) / kMinTokChunk) +
-                  (Is > 0 ? (B + kMinTokChunk - 1) / kMinTokChunk : 0);
+  L.max_entries = max_entries_for(B, E, k, Is);
   L.ctrl = take(kCtrlWords * 4 + kTraceSteps * kTrSlots * 8);
   L.topk_idx = take(slots * 4);
   L.topk_gate = take(slots * 4);
@@ -329,6 +334,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map,
       "tx::bytes.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar), "l"(policy)
       : "memory");
+}
+// L2 prefetch of one box of a 2-D tensor map (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_2d(const void *map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   (uint64_t)map),
+               "r"(x), "r"(y)
+               : "memory");
 }
 __device__ __forceinline__ void prefetch_l2(const void *p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));

@@ -224,6 +224,30 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
+  // While the grouping kernel runs (this grid may already be resident), warm
+  // L2 with this CTA's likely first work item: the gate/up tile that item
+  // number blockIdx.x had in the previous call's work list, which is still in
+  // the workspace (or being rewritten).  Prefetches only, every index bounded,
+  // so a wrong guess costs bandwidth, never correctness.
+  if constexpr (!kShared) {
+    if (warp == 0 && lane == 0) {
+      const int t1g = d.I / kGateRows;
+      const int entry = blockIdx.x / t1g;
+      const int n_prev = __ldcg(&ws.ctrl[kCtrlNumEntries]);
+      if (entry < n_prev && entry < max_entries_for(d.B, d.E, d.k, d.Is)) {
+        const int e = __ldcg(&ws.entries[entry]).x;
+        if (e >= 0 && e < d.E) {
+          const int row0 = e * 2 * d.I + (blockIdx.x - entry * t1g) * kGateRows;
+          const int nk = min(stages, d.H / kBlockK);
+          for (int kc = 0; kc < nk; ++kc) {
+            tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0);
+            tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + d.I);
+          }
+        }
+      }
+    }
+  }
+
   // Everything below reads the grouping kernel's results.
   pdl_wait_primary();
 #ifdef SLIMWISE_TRACE
