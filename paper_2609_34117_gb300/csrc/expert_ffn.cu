@@ -238,8 +238,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         const int e = __ldcg(&ws.entries[entry]).x;
         if (e >= 0 && e < d.E) {
           const int row0 = e * 2 * d.I + (blockIdx.x - entry * t1g) * kGateRows;
-          const int nk = min(stages, d.H / kBlockK);
-          for (int kc = 0; kc < nk; ++kc) {
+          for (int kc = 0; kc < d.H / kBlockK; ++kc) {
             tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0);
             tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + d.I);
           }
