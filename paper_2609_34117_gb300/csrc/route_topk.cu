@@ -81,6 +81,7 @@ struct StageType<4> {
   using T = __nv_bfloat16;
 };
 
+
 // Shared memory of one CTA: hidden rows [TB][H] (StageType), logits of its
 // slice [TB][slice] fp32, retained ids [m] int32.  Rows of tokens past the
 // batch are zero, so every token slot computes (and discards) a logit.
@@ -222,9 +223,11 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   }
   cluster.sync();  // every slice's logits are visible cluster-wide
 
-  // Top-k and gates: warp w of CTA 0 handles token w of the cluster.
-  if (crank == 0 && warp < nt) {
-    const int t = t0 + warp;
+  // Top-k and gates: token tw of the cluster is handled by warp tw / 8 of the
+  // cluster's CTA tw % 8, so the tokens' top-k run side by side.
+  const int tw = warp * kClusterCtas + crank;
+  if (tw < nt) {
+    const int t = t0 + tw;
     float my_z = 0.0f;
     int my_e = 0;
     if constexpr (NC > 0) {
@@ -238,7 +241,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
         const int r = lane + 32 * i;
         if (r < m) {
           const int owner = r / slice;
-          zc[i] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
+          zc[i] = cluster.map_shared_rank(zs, owner)[(size_t)tw * slice + (r - owner * slice)];
         }
       }
       unsigned long long key[NC];
@@ -282,7 +285,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
           const int r = r0 + 32 * u;
           if (r < m) {
             const int owner = r / slice;
-            zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)warp * slice + (r - owner * slice)];
+            zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)tw * slice + (r - owner * slice)];
           }
         }
 #pragma unroll
