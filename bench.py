@@ -374,34 +374,64 @@ def graph_measure(sw, layer, B, point, calls=20, reps=50):
 
 
 def e2e_measure(sw, layer, B, m_prime, steps, device, point):
-    """Same metric through the C ABI with host buffers: pinned H2D of the batch,
-    the layer, D2H of the output, all inside the timed region."""
+    """Same metric through the C ABI with host buffers: every step copies its
+    batch from pinned host memory to the device, runs the layer and copies the
+    output back, all inside the timed region.  As a serving loop would, the
+    copies run on a copy stream with two device buffers each way, so the
+    input of step i+1 and the output of step i move while step i computes."""
     shape = layer.shape
     batches, retained, ws_buf, out, copy_for_step = point["_state"]
     host_in = [b.cpu().pin_memory() for b in batches]
-    host_out = torch.empty((B, shape.hidden), dtype=torch.bfloat16).pin_memory()
-    dev_in = torch.empty_like(batches[0])
-    stream = torch.cuda.current_stream()
-    k = shape.top_k
+    host_out = [torch.empty((B, shape.hidden), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    dev_in = [torch.empty_like(batches[0]) for _ in range(2)]
+    dev_out = [torch.empty_like(out) for _ in range(2)]
+    st = torch.cuda.current_stream()
+    cs = torch.cuda.Stream(device=device)
+    ev = lambda: torch.cuda.Event()  # noqa: E731
+    ev_in, ev_done, ev_out = [ev(), ev()], [ev(), ev()], [ev(), ev()]
 
-    def one(i):
-        dev_in.copy_(host_in[i % len(host_in)], non_blocking=True)
+    def h2d(i):
+        j = i % 2
+        cs.wait_event(ev_done[j])           # the layer that read dev_in[j] is done
+        with torch.cuda.stream(cs):
+            dev_in[j].copy_(host_in[i % len(host_in)], non_blocking=True)
+        ev_in[j].record(cs)
+
+    def layer_step(i):
+        j = i % 2
+        st.wait_event(ev_in[j])             # this step's batch is on the device
+        st.wait_event(ev_out[j])            # dev_out[j] was copied out
         w_gu, w_d = layer.copies[copy_for_step(i)]
-        layer.call(sw, dev_in, retained, w_gu, w_d, out, ws_buf, stream)
-        host_out.copy_(out, non_blocking=True)
+        layer.call(sw, dev_in[j], retained, w_gu, w_d, dev_out[j], ws_buf, st)
+        ev_done[j].record(st)
 
-    for i in range(5):
-        one(i)
+    def d2h(i):
+        j = i % 2
+        cs.wait_event(ev_done[j])
+        with torch.cuda.stream(cs):
+            host_out[j].copy_(dev_out[j], non_blocking=True)
+        ev_out[j].record(cs)
+
+    def run(n):
+        h2d(0)
+        for i in range(n):
+            if i + 1 < n:
+                h2d(i + 1)
+            layer_step(i)
+            d2h(i)
+
+    run(5)
     torch.cuda.synchronize()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for i in range(steps):
-        one(i)
-    t1.record(stream)
+    t0.record(cs)                           # before the first input copy
+    run(steps)
+    st.wait_stream(cs)                      # after the last output copy
+    t1.record(st)
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1) / steps
     return {"value": B / (ms * 1e-3), "unit": "tokens/s", "ms_per_step": ms,
-            "h2d_bytes_per_step": B * shape.hidden * 2, "d2h_bytes_per_step": B * shape.hidden * 2}
+            "h2d_bytes_per_step": B * shape.hidden * 2, "d2h_bytes_per_step": B * shape.hidden * 2,
+            "copies": "pinned host buffers, copy stream overlapped with compute (double-buffered)"}
 
 
 def cpu_baseline(layer, B, m_prime, budget_s=15.0):
