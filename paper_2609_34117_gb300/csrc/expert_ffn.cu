@@ -651,14 +651,16 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   int optin = 0;
   err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (err != cudaSuccess) return err;
-  // leave room on each SM for the next layer's routing CTAs, which become
-  // resident while this grid finishes (programmatic dependent launch)
   // the token maps exist for boxes of 16 << m <= tok_chunk rows, and an
   // entry's box covers at most tok_chunk rows: tok_chunk must be a power of
   // two in [16, 256]
   if (d.tok_chunk < kTokBox || d.tok_chunk > kMaxTokTile || (d.tok_chunk & (d.tok_chunk - 1)))
     return cudaErrorInvalidValue;
-  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - kCoResidentSmem);
+  // leave room on each SM for the next layer's routing CTAs, which become
+  // resident while this grid finishes (programmatic dependent launch), where
+  // they can fit at all: routing CTAs of 8 tokens never do
+  const size_t reserve = route_tokens_per_cluster(d.B) <= 4 ? kCoResidentSmem : 0;
+  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - reserve);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
   auto kernel = d.Is > 0 ? expert_ffn_kernel<true> : expert_ffn_kernel<false>;

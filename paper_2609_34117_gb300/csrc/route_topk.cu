@@ -31,6 +31,7 @@ constexpr int kRouteThreads = 256;
 constexpr int kRouteWarps = kRouteThreads / 32;
 constexpr int kClusterCtas = 8;
 constexpr int kChunkBatch = 8;  // 128-wide chunks whose loads are issued together
+constexpr int kPairChunkBatch = 4;  // the same, per row, when a warp takes two rows
 
 // Order-preserving map of an fp32 value to uint32 (-0 folded onto +0).
 __device__ __forceinline__ uint32_t logit_order_bits(float z) {
@@ -65,6 +66,24 @@ __device__ __forceinline__ void fma_chunk(const XT *xs, int H, int col, float4 w
     p[t] = fmaf(x.y, w.y, p[t]);
     p[t] = fmaf(x.z, w.z, p[t]);
     p[t] = fmaf(x.w, w.w, p[t]);
+  }
+}
+
+// Two router rows at once: each staged hidden vector feeds both rows' sums.
+template <int TB, typename XT>
+__device__ __forceinline__ void fma_chunk2(const XT *xs, int H, int col, float4 w0, float4 w1,
+                                           float (&p0)[TB], float (&p1)[TB]) {
+#pragma unroll
+  for (int t = 0; t < TB; ++t) {
+    const float4 x = load_x4(xs, (size_t)t * H + col);
+    p0[t] = fmaf(x.x, w0.x, p0[t]);
+    p0[t] = fmaf(x.y, w0.y, p0[t]);
+    p0[t] = fmaf(x.z, w0.z, p0[t]);
+    p0[t] = fmaf(x.w, w0.w, p0[t]);
+    p1[t] = fmaf(x.x, w1.x, p1[t]);
+    p1[t] = fmaf(x.y, w1.y, p1[t]);
+    p1[t] = fmaf(x.z, w1.z, p1[t]);
+    p1[t] = fmaf(x.w, w1.w, p1[t]);
   }
 }
 
@@ -177,28 +196,80 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   }
 
   // Hidden rows of the cluster's tokens (16-byte vectors of 8 bf16), zero
-  // past the batch.
+  // past the batch.  Each thread issues TB loads before storing any, so the
+  // staging costs one memory round trip per TB * 256 vectors.
   const int vecs = H / 8;
-  for (int i = threadIdx.x; i < TB * vecs; i += blockDim.x) {
-    const int t = i / vecs, v = i - t * vecs;
-    const uint4 raw = t < nt ? reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v]
-                             : make_uint4(0u, 0u, 0u, 0u);
-    if constexpr (sizeof(XT) == 2) {
-      reinterpret_cast<uint4 *>(xs)[(size_t)t * vecs + v] = raw;
-    } else {
-      float4 *dst = reinterpret_cast<float4 *>(xs + (size_t)t * H + 8 * v);
-      dst[0] = make_float4(__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xFFFF0000u),
-                           __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xFFFF0000u));
-      dst[1] = make_float4(__uint_as_float(raw.z << 16), __uint_as_float(raw.z & 0xFFFF0000u),
-                           __uint_as_float(raw.w << 16), __uint_as_float(raw.w & 0xFFFF0000u));
+  for (int i0 = 0; i0 < TB * vecs; i0 += TB * kRouteThreads) {
+    uint4 raw[TB];
+#pragma unroll
+    for (int u = 0; u < TB; ++u) {
+      const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
+      const int t = i / vecs, v = i - t * vecs;
+      raw[u] = (i < TB * vecs && t < nt)
+                   ? reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v]
+                   : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int u = 0; u < TB; ++u) {
+      const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
+      if (i >= TB * vecs) break;
+      const int t = i / vecs, v = i - t * vecs;
+      if constexpr (sizeof(XT) == 2) {
+        reinterpret_cast<uint4 *>(xs)[(size_t)t * vecs + v] = raw[u];
+      } else {
+        float4 *dst = reinterpret_cast<float4 *>(xs + (size_t)t * H + 8 * v);
+        dst[0] = make_float4(__uint_as_float(raw[u].x << 16), __uint_as_float(raw[u].x & 0xFFFF0000u),
+                             __uint_as_float(raw[u].y << 16), __uint_as_float(raw[u].y & 0xFFFF0000u));
+        dst[1] = make_float4(__uint_as_float(raw[u].z << 16), __uint_as_float(raw[u].z & 0xFFFF0000u),
+                             __uint_as_float(raw[u].w << 16), __uint_as_float(raw[u].w & 0xFFFF0000u));
+      }
     }
   }
   __syncthreads();
 
-  // Logits of this CTA's slice [r_lo, r_hi) of the retained list.
+  // Logits of this CTA's slice [r_lo, r_hi) of the retained list.  With at
+  // least two rows per warp, a warp takes its rows in pairs (rows r, r + 1),
+  // which halves the shared-memory reads of the staged hidden rows; the sums
+  // and their order are those of one row at a time.
   const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
   const int nchunks = H / 128;
-  for (int r = r_lo + warp; r < r_hi; r += kRouteWarps) {
+  const int npair = (r_hi - r_lo >= 2 * kRouteWarps) ? (r_hi - r_lo) / 2 : 0;
+  for (int pi = warp; pi < npair; pi += kRouteWarps) {
+    const int r = r_lo + 2 * pi;
+    const float4 *w0 = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r] * H) + lane;
+    const float4 *w1 = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r + 1] * H) + lane;
+    float p0[TB], p1[TB];
+#pragma unroll
+    for (int t = 0; t < TB; ++t) p0[t] = p1[t] = 0.0f;
+    for (int c0 = 0; c0 < nchunks; c0 += kPairChunkBatch) {
+      float4 v0[kPairChunkBatch], v1[kPairChunkBatch];
+#pragma unroll
+      for (int u = 0; u < kPairChunkBatch; ++u)
+        if (c0 + u < nchunks) {
+          v0[u] = __ldg(w0 + 32 * (c0 + u));
+          v1[u] = __ldg(w1 + 32 * (c0 + u));
+        }
+#pragma unroll
+      for (int u = 0; u < kPairChunkBatch; ++u)
+        if (c0 + u < nchunks)
+          fma_chunk2<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v0[u], v1[u], p0, p1);
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1)
+#pragma unroll
+      for (int t = 0; t < TB; ++t) {
+        p0[t] = p0[t] + __shfl_xor_sync(0xFFFFFFFFu, p0[t], off);
+        p1[t] = p1[t] + __shfl_xor_sync(0xFFFFFFFFu, p1[t], off);
+      }
+    if (lane == 0)
+#pragma unroll
+      for (int t = 0; t < TB; ++t)
+        if (t < nt) {
+          zs[(size_t)t * slice + (r - r_lo)] = p0[t];
+          zs[(size_t)t * slice + (r + 1 - r_lo)] = p1[t];
+        }
+  }
+  for (int r = r_lo + 2 * npair + warp; r < r_hi; r += kRouteWarps) {
     const float4 *wrow = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r] * H) + lane;
     float p[TB];
 #pragma unroll
@@ -372,10 +443,12 @@ cudaError_t launch_route_nc(const __nv_bfloat16 *hidden, const float *router_w,
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
                               const int32_t *retained, Dims d, Ws ws, bool pdl,
                               cudaStream_t stream) {
-  if (d.B <= 32) return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
-  if (d.B <= 64) return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
-  if (d.B <= 256) return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);
-  return launch_route_nc<8>(hidden, router_w, retained, d, ws, pdl, stream);
+  switch (route_tokens_per_cluster(d.B)) {
+    case 1: return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
+    case 2: return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
+    case 4: return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);
+    default: return launch_route_nc<8>(hidden, router_w, retained, d, ws, pdl, stream);
+  }
 }
 
 }  // namespace slimwise
