@@ -70,6 +70,9 @@ enum CtrlWord {
   kCtrlWorkCounter = 4, // dynamic scheduler counter
   kCtrlErr = 5,         // SLIMWISE_DEVERR_* bits of the current call
   kCtrlTraceStep = 6,   // step counter of the optional trace ring
+  kCtrlCombTail = 7,    // (token, h tile) combines queued by the FFN kernel
+  kCtrlCombHead = 8,    // queue slots taken by combining warps
+  kCtrlDownDone = 9,    // down items whose epilogue has finished
   kCtrlWords = 16
 };
 
@@ -85,7 +88,7 @@ enum TraceSlot {
 // Byte offsets of every workspace region (all 1024-byte aligned).
 struct WsLayout {
   size_t ctrl, topk_idx, topk_gate, counts, offsets, union_ids, entries,
-      entry_done, perm, pos, comb_cnt, xp, act, y, shared_gate, xt, act_s, y_s, total;
+      entry_done, perm, pos, comb_cnt, comb_q, xp, act, y, shared_gate, xt, act_s, y_s, total;
   int32_t max_entries;
 };
 
@@ -124,6 +127,7 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
   L.perm = take(slots * 4);
   L.pos = take(slots * 4);
   L.comb_cnt = take((size_t)B * (H / kCombineTile) * 4);
+  L.comb_q = take((size_t)B * (H / kCombineTile) * 4);
   L.xp = take(slots * H * 2);
   L.act = take(slots * I * 2);
   L.y = take(slots * H * 4);
@@ -152,6 +156,7 @@ struct Ws {
   int32_t *perm;
   int32_t *pos;
   int32_t *comb_cnt;   // [B, H/128] down items finished per (token, h tile)
+  int32_t *comb_q;     // [B * H/128] queued combines, 1 + t * (H/128) + tile; 0 = empty
   __nv_bfloat16 *xp;   // [B*k, H] hidden rows in grouped order
   __nv_bfloat16 *act;  // [B*k, I] SwiGLU activations in grouped order
   float *y;            // [B*k, H] expert outputs in grouped order
@@ -175,6 +180,7 @@ inline Ws make_ws(void *base, const WsLayout &L) {
   w.perm = (int32_t *)(b + L.perm);
   w.pos = (int32_t *)(b + L.pos);
   w.comb_cnt = (int32_t *)(b + L.comb_cnt);
+  w.comb_q = (int32_t *)(b + L.comb_q);
   w.xp = (__nv_bfloat16 *)(b + L.xp);
   w.act = (__nv_bfloat16 *)(b + L.act);
   w.y = (float *)(b + L.y);

@@ -44,8 +44,11 @@ constexpr int kItemRing = 4;
 constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
 constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
 constexpr int kEpiWarps = kEpiThreads / 32;
-// per epilogue group: combine count and token list
-constexpr int kGroupMiscInts = 1 + kMaxTokTile;
+// per epilogue group: combine count, queue base and token list
+constexpr int kGroupMiscInts = 2 + kMaxTokTile;
+// tokens a down item's epilogue combines itself; the rest of its list goes
+// to the grid-wide combine queue
+constexpr int kInlineCombines = 2 * kEpiThreads / 32;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 // 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
@@ -137,6 +140,67 @@ __device__ __forceinline__ Item decode_item(int item, const ItemPlan &ip, const 
   return it;
 }
 
+// out[t, h] = sum_j g[t,j] y[pos(t,j), h] in j order (then the shared
+// expert's term) for the 128 h of one tile, by one warp: lane l covers
+// h = 4l..4l+3 with one 16-byte load per selection (a y tile row is 512
+// contiguous bytes), up to 8 loads in flight per lane; lanes j < k hold
+// selection j's grouped position and gate.
+template <bool kShared>
+__device__ __forceinline__ void combine_token(const Ws &ws, const Dims &d,
+                                              __nv_bfloat16 *__restrict__ out, int t, int tile,
+                                              int lane) {
+  const float *ytile = ws.y + tile * kCombineTile + 4 * lane;
+  int p = 0;
+  float gj = 0.0f;
+  if (lane < d.k) {
+    p = __ldcg(&ws.pos[(size_t)t * d.k + lane]);
+    gj = __ldcg(&ws.topk_gate[(size_t)t * d.k + lane]);
+  }
+  float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  for (int j0 = 0; j0 < d.k; j0 += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      const int pj = __shfl_sync(0xFFFFFFFFu, p, (j0 + jj) & 31);
+      if (j0 + jj < d.k)
+        v[jj] = __ldcg(reinterpret_cast<const float4 *>(ytile + (size_t)pj * d.H));
+    }
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      const float w = __shfl_sync(0xFFFFFFFFu, gj, (j0 + jj) & 31);
+      if (j0 + jj < d.k) {
+        acc.x = fmaf(w, v[jj].x, acc.x);
+        acc.y = fmaf(w, v[jj].y, acc.y);
+        acc.z = fmaf(w, v[jj].z, acc.z);
+        acc.w = fmaf(w, v[jj].w, acc.w);
+      }
+    }
+  }
+  if constexpr (kShared) {
+    // the shared expert's term, after the k routed ones (Sec. 3.3)
+    const float sg = __ldcg(&ws.shared_gate[t]);
+    const float4 vs = __ldcg(reinterpret_cast<const float4 *>(
+        ws.y_s + (size_t)t * d.H + tile * kCombineTile + 4 * lane));
+    acc.x = fmaf(sg, vs.x, acc.x);
+    acc.y = fmaf(sg, vs.y, acc.y);
+    acc.z = fmaf(sg, vs.z, acc.z);
+    acc.w = fmaf(sg, vs.w, acc.w);
+  }
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
+  *reinterpret_cast<uint2 *>(out + (size_t)t * d.H + tile * kCombineTile + 4 * lane) =
+      make_uint2(*reinterpret_cast<const uint32_t *>(&lo),
+                 *reinterpret_cast<const uint32_t *>(&hi));
+}
+
+// The combine queue pays where the combine lists are long, at 32 or more
+// tokens per retained expert on average; below that its end-of-launch
+// handshake (the last down item closes the queue, the waiting warps see it)
+// costs more than the combines it spreads.
+__device__ __forceinline__ bool use_combine_queue(const Dims &d) {
+  return d.B * d.k >= 32 * d.m_ret;
+}
+
 // Named barrier of epilogue group g (ids 1.., id 0 is __syncthreads).
 __device__ __forceinline__ void epi_bar(int g) {
   asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kEpiThreads) : "memory");
@@ -153,8 +217,11 @@ __device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit
   atomicOr(&ws.ctrl[kCtrlErr], bit);
 }
 
+// At most 128 registers a thread (320 threads: 40 K of the SM's 64 K), so
+// that a routing CTA of the next layer (256 threads, at most 96 registers)
+// can become resident beside this one.
 template <bool kShared>
-__global__ void __launch_bounds__(kFfnThreads, 1)
+__global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
                       int tmem_cols) {
@@ -461,8 +528,12 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     float *xb = xch + g * kTileRows * kXchStride;
     int *gm = group_misc + g * kGroupMiscInts;
     int *comb_n = gm;
-    int *comb_list = gm + 1;                          // [kMaxTokTile]
+    int *q_base = gm + 1;
+    int *comb_list = gm + 2;                          // [kMaxTokTile]
     const int ew = q;                                 // warp within the group
+    const int total_down = total - ip.r1 - ip.S * ip.t1s;  // down items of the launch
+    const int q_cap = d.B * t2;                            // combine-queue slots
+    const bool comb_queue = use_combine_queue(d);
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
@@ -561,59 +632,71 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         __threadfence();
         epi_bar(g);
         const int n_list = *comb_n;
-        // out[t, h] = sum_j g[t,j] y[pos(t,j), h] in j order, for the 128 h
-        // of this tile.  A warp takes one token at a time: lane l covers
-        // h = 4l..4l+3 with one 16-byte load per selection (a y tile row is
-        // 512 contiguous bytes), up to 8 loads in flight per lane; lanes
-        // j < k hold selection j's grouped position and gate.
-        const float *ytile = ws.y + it.tile * kCombineTile + 4 * lane;
-        for (int i = ew; i < n_list; i += kEpiWarps) {
-          const int t = comb_list[i];
-          int p = 0;
-          float gj = 0.0f;
-          if (lane < d.k) {
-            p = __ldcg(&ws.pos[(size_t)t * d.k + lane]);
-            gj = __ldcg(&ws.topk_gate[(size_t)t * d.k + lane]);
-          }
-          float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-          for (int j0 = 0; j0 < d.k; j0 += 8) {
-            float4 v[8];
-#pragma unroll
-            for (int jj = 0; jj < 8; ++jj) {
-              const int pj = __shfl_sync(0xFFFFFFFFu, p, (j0 + jj) & 31);
-              if (j0 + jj < d.k)
-                v[jj] = __ldcg(reinterpret_cast<const float4 *>(ytile + (size_t)pj * d.H));
-            }
-#pragma unroll
-            for (int jj = 0; jj < 8; ++jj) {
-              const float w = __shfl_sync(0xFFFFFFFFu, gj, (j0 + jj) & 31);
-              if (j0 + jj < d.k) {
-                acc.x = fmaf(w, v[jj].x, acc.x);
-                acc.y = fmaf(w, v[jj].y, acc.y);
-                acc.z = fmaf(w, v[jj].z, acc.z);
-                acc.w = fmaf(w, v[jj].w, acc.w);
-              }
-            }
-          }
-          if constexpr (kShared) {
-            // the shared expert's term, after the k routed ones (Sec. 3.3)
-            const float sg = __ldcg(&ws.shared_gate[t]);
-            const float4 vs = __ldcg(reinterpret_cast<const float4 *>(
-                ws.y_s + (size_t)t * d.H + it.tile * kCombineTile + 4 * lane));
-            acc.x = fmaf(sg, vs.x, acc.x);
-            acc.y = fmaf(sg, vs.y, acc.y);
-            acc.z = fmaf(sg, vs.z, acc.z);
-            acc.w = fmaf(sg, vs.w, acc.w);
-          }
-          const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
-          const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
-          *reinterpret_cast<uint2 *>(out + (size_t)t * d.H + it.tile * kCombineTile + 4 * lane) =
-              make_uint2(*reinterpret_cast<const uint32_t *>(&lo),
-                         *reinterpret_cast<const uint32_t *>(&hi));
+        // With the combine queue, the first kInlineCombines tokens of the
+        // list are combined here and the rest go to the grid-wide queue,
+        // which every epilogue group drains once it has no items left: the
+        // last experts' items complete most tokens, and their lists would
+        // otherwise be combined one warp round trip at a time on a few CTAs
+        // after all streaming has ended.
+        const int n_inline = comb_queue ? min(n_list, kInlineCombines) : n_list;
+        if (n_list > n_inline) {
+          if (et == 0) *q_base = atomicAdd(&ws.ctrl[kCtrlCombTail], n_list - n_inline);
+          epi_bar(g);
+          const int base = *q_base;
+          // each (token, tile) completes once per call: at most B * t2 slots
+          for (int i = n_inline + et; i < n_list; i += kEpiThreads)
+            if (base + (i - n_inline) < q_cap)
+              ws.comb_q[base + (i - n_inline)] = 1 + comb_list[i] * t2 + it.tile;
+          __threadfence();
         }
-        // comb_list and comb_n are reused by this group's next down item
+        for (int i = ew; i < n_inline; i += kEpiWarps)
+          combine_token<kShared>(ws, d, out, comb_list[i], it.tile, lane);
+        // comb_list and comb_n are reused by this group's next down item.
+        // The queued combines are published before the item counts as done;
+        // the launch's last down item then knows the final queue length and
+        // closes every slot past it (-1), which ends the waits below.
         epi_bar(g);
+        if (comb_queue) {
+          if (et == 0) {
+            __threadfence();
+            const int done = atomicAdd(&ws.ctrl[kCtrlDownDone], 1) + 1;
+            *q_base = done == total_down ? ld_acquire(&ws.ctrl[kCtrlCombTail]) : -1;
+          }
+          epi_bar(g);
+          const int q_final = *q_base;
+          if (q_final >= 0)
+            for (int i = q_final + et; i < q_cap; i += kEpiThreads) ws.comb_q[i] = -1;
+        }
       }
+    }
+    // No items left for this group: take queued combines, each warp one slot
+    // at a time, until it draws a closed slot.
+    while (comb_queue && !*abort && total_down > 0) {
+      int v = -1;
+      if (lane == 0) {
+        const int h = atomicAdd(&ws.ctrl[kCtrlCombHead], 1);
+        if (h < q_cap) {
+          const uint64_t t0 = global_timer_ns();
+          uint32_t nap = 64;
+          for (;;) {
+            const int x = ld_acquire(&ws.comb_q[h]);
+            if (x != 0) {
+              v = x;
+              break;
+            }
+            if (*abort) break;
+            if (global_timer_ns() - t0 > kTimeoutNs) {
+              raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
+              break;
+            }
+            __nanosleep(nap);
+            if (nap < 1024) nap <<= 1;
+          }
+        }
+      }
+      v = __shfl_sync(0xFFFFFFFFu, v, 0);
+      if (v <= 0 || v > q_cap) break;
+      combine_token<kShared>(ws, d, out, (v - 1) / t2, (v - 1) % t2, lane);
     }
   }
 

@@ -329,6 +329,26 @@ def test_workspace_contents_do_not_matter(tiny):
     assert sw.slimwise_moe_device_status(ws) == 0
 
 
+@pytest.mark.parametrize("fill", [0xFF, 0x00])
+def test_long_combine_lists_all_outputs(tiny, fill):
+    # 600 tokens, k = 4 of m' = 8: 300 tokens per retained expert, two work
+    # entries each, so most (token, h tile) combines are completed by items
+    # with long lists and go through the grid-wide combine queue; a workspace
+    # of 0xFF bytes (queue slots reading as closed) must not change anything
+    shape = tiny.shape
+    B, k = 600, 4
+    x = synth.hidden_states(B, shape, 21)
+    retained = synth.retained_set(shape.num_experts, 8, 5)
+    ws = sw.alloc_workspace(B, shape.hidden, shape.num_experts, shape.inter, k, DEV)
+    ws.fill_(fill)
+    out = sw.slimwise_moe_decode(x.to(DEV), tiny.d_wr, retained.to(DEV), tiny.d_w_gu, tiny.d_w_d,
+                                 k, workspace=ws)
+    torch.cuda.synchronize()
+    assert sw.slimwise_moe_device_status(ws) == 0
+    ref = _oracle(tiny, x, retained, k)
+    _check_out(out.float().cpu().numpy(), ref["out"])
+
+
 def test_duplicate_retained_id_is_reported(tiny):
     shape = tiny.shape
     x = synth.hidden_states(4, shape, 4).to(DEV)
