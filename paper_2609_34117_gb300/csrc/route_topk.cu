@@ -4,11 +4,11 @@
 //
 // A thread-block cluster of kClusterCtas CTAs handles TB tokens.  CTA r of
 // the cluster evaluates the logits of its slice of the retained experts for
-// those tokens and keeps them in its shared memory; after a cluster barrier
-// the warps of CTA 0 run the top-k of each token over all slices, reading the
-// other CTAs' logits through distributed shared memory.  Each CTA thus reads
-// only 1/kClusterCtas of the router rows, and no global counter or second
-// kernel is needed to join the slices.
+// those tokens and writes each one, through distributed shared memory, into
+// the shared memory of the CTA that runs that token's top-k (token tw on CTA
+// tw mod 8); after one cluster barrier every top-k reads only its own shared
+// memory.  Each CTA thus reads only 1/kClusterCtas of the router rows, and no
+// global counter or second kernel is needed to join the slices.
 //
 // Logits follow the canonical fp32 order: lane l of a warp owns elements
 // 128c + 4l + q (q = 0..3) of every 128-wide chunk c, accumulated with fused
@@ -101,9 +101,10 @@ struct StageType<4> {
 };
 
 
-// Shared memory of one CTA: hidden rows [TB][H] (StageType), logits of its
-// slice [TB][slice] fp32, retained ids [m] int32.  Rows of tokens past the
-// batch are zero, so every token slot computes (and discards) a logit.
+// Shared memory of one CTA: hidden rows [TB][H] (StageType), the logits of
+// the tokens whose top-k it runs [ceil(TB/8)][m] fp32 (written by every CTA
+// of the cluster), retained ids [m] int32.  Rows of tokens past the batch are
+// zero, so every token slot computes (and discards) a logit.
 // Round j of the top-k: the winner (order bits whi, complemented id wlo) goes
 // to lane j.  With no candidate left (fewer than k distinct ids, already
 // reported) a valid id stands in.
@@ -133,9 +134,10 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   const int crank = (int)cluster.block_rank();
   const int H = d.H, m = d.m_ret, k = d.k;
   const int slice = (m + kClusterCtas - 1) / kClusterCtas;
+  constexpr int kOwn = (TB + kClusterCtas - 1) / kClusterCtas;  // tokens whose top-k a CTA runs
   XT *xs = reinterpret_cast<XT *>(smem);
-  float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * sizeof(XT));
-  int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)TB * slice);
+  float *zs = reinterpret_cast<float *>(smem + (size_t)TB * H * sizeof(XT));  // [kOwn][m]
+  int32_t *ids = reinterpret_cast<int32_t *>(zs + (size_t)kOwn * m);
 
   // Before waiting for the previous kernel on the stream (this CTA may be
   // resident while it finishes): warm L2 with this CTA's router rows.  These
@@ -261,13 +263,14 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
         p0[t] = p0[t] + __shfl_xor_sync(0xFFFFFFFFu, p0[t], off);
         p1[t] = p1[t] + __shfl_xor_sync(0xFFFFFFFFu, p1[t], off);
       }
-    if (lane == 0)
+    // lane t sends token t's two logits to the CTA that runs its top-k
 #pragma unroll
-      for (int t = 0; t < TB; ++t)
-        if (t < nt) {
-          zs[(size_t)t * slice + (r - r_lo)] = p0[t];
-          zs[(size_t)t * slice + (r + 1 - r_lo)] = p1[t];
-        }
+    for (int t = 0; t < TB; ++t)
+      if (lane == t && t < nt) {
+        float *dst = cluster.map_shared_rank(zs, t % kClusterCtas) + (size_t)(t / kClusterCtas) * m;
+        dst[r] = p0[t];
+        dst[r + 1] = p1[t];
+      }
   }
   for (int r = r_lo + 2 * npair + warp; r < r_hi; r += kRouteWarps) {
     const float4 *wrow = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r] * H) + lane;
@@ -287,12 +290,14 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
     for (int off = 16; off >= 1; off >>= 1)
 #pragma unroll
       for (int t = 0; t < TB; ++t) p[t] = p[t] + __shfl_xor_sync(0xFFFFFFFFu, p[t], off);
-    if (lane == 0)
 #pragma unroll
-      for (int t = 0; t < TB; ++t)
-        if (t < nt) zs[(size_t)t * slice + (r - r_lo)] = p[t];
+    for (int t = 0; t < TB; ++t)
+      if (lane == t && t < nt)
+        cluster.map_shared_rank(zs, t % kClusterCtas)[(size_t)(t / kClusterCtas) * m + r] = p[t];
   }
-  cluster.sync();  // every slice's logits are visible cluster-wide
+  // every logit is in the shared memory of the CTA that needs it; after this
+  // barrier no CTA touches another's shared memory, so none waits at the end
+  cluster.sync();
 
   // Top-k and gates: token tw of the cluster is handled by warp tw / 8 of the
   // cluster's CTA tw % 8, so the tokens' top-k run side by side.
@@ -305,14 +310,13 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
       // this lane's candidates r = lane + 32 i (i < NC) as 64-bit keys
       // (order-preserving logit bits, complemented id; 0 = none), kept sorted
       // descending in registers -- every index below is a compile-time one;
-      // all remote loads are issued before any is used
+      // all loads are issued before any is used
       float zc[NC];
 #pragma unroll
       for (int i = 0; i < NC; ++i) {
         const int r = lane + 32 * i;
         if (r < m) {
-          const int owner = r / slice;
-          zc[i] = cluster.map_shared_rank(zs, owner)[(size_t)tw * slice + (r - owner * slice)];
+          zc[i] = zs[(size_t)warp * m + r];
         }
       }
       unsigned long long key[NC];
@@ -355,8 +359,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
         for (int u = 0; u < 4; ++u) {
           const int r = r0 + 32 * u;
           if (r < m) {
-            const int owner = r / slice;
-            zc[u] = cluster.map_shared_rank(zs, owner)[(size_t)tw * slice + (r - owner * slice)];
+            zc[u] = zs[(size_t)warp * m + r];
           }
         }
 #pragma unroll
@@ -395,7 +398,6 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
       ws.topk_gate[(size_t)t * k + lane] = w / denom;
     }
   }
-  cluster.sync();  // keep every CTA's shared memory alive until CTA 0 is done
 #ifdef SLIMWISE_TRACE
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     trace_stamp(ws, tr_step, kTrRouteEnd);
@@ -408,9 +410,9 @@ template <int TB, int NC>
 cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
                             const int32_t *retained, Dims d, Ws ws, bool pdl,
                             cudaStream_t stream) {
-  const int slice = (d.m_ret + kClusterCtas - 1) / kClusterCtas;
   const size_t smem = (size_t)TB * d.H * sizeof(typename StageType<TB>::T) +
-                      (size_t)TB * slice * 4 + (size_t)d.m_ret * 4;
+                      (size_t)((TB + kClusterCtas - 1) / kClusterCtas) * d.m_ret * 4 +
+                      (size_t)d.m_ret * 4;
   cudaError_t err = cudaFuncSetAttribute(
       route_topk_kernel<TB, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
