@@ -24,7 +24,7 @@
 
 namespace slimwise {
 
-constexpr int kGroupTokens = 4;
+constexpr int kGroupTokens = 2;
 constexpr int kGroupThreads = 512;
 
 // Exclusive scan of vals[0..n) (n <= kMaxExperts) into outp[0..n], by one
@@ -102,15 +102,29 @@ __global__ void __launch_bounds__(kGroupThreads)
   if (tid == 0) bad = 0;
   __syncthreads();
   const int nslots = nt * k;
-  for (int s = tid; s < S; s += blockDim.x) {
-    int e = ws.topk_idx[s];
-    if (e < 0 || e >= E) {  // only possible for caller-given selections
-      bad = SLIMWISE_DEVERR_BAD_TOPK;
-      e = min(max(e, 0), E - 1);
+  // each thread's selections are loaded together, then counted
+  constexpr int kHistBatch = 8;
+  for (int s0 = tid; s0 < S; s0 += kHistBatch * blockDim.x) {
+    int ev[kHistBatch];
+#pragma unroll
+    for (int u = 0; u < kHistBatch; ++u) {
+      const int s = s0 + u * blockDim.x;
+      ev[u] = s < S ? ws.topk_idx[s] : 0;
     }
-    atomicAdd(&cnt_all[e], 1);
-    if (s < t0 * k) atomicAdd(&cnt_before[e], 1);
-    else if (s < t1 * k) my_ids[s - t0 * k] = e;
+#pragma unroll
+    for (int u = 0; u < kHistBatch; ++u) {
+      const int s = s0 + u * blockDim.x;
+      if (s < S) {
+        int e = ev[u];
+        if (e < 0 || e >= E) {  // only possible for caller-given selections
+          bad = SLIMWISE_DEVERR_BAD_TOPK;
+          e = min(max(e, 0), E - 1);
+        }
+        atomicAdd(&cnt_all[e], 1);
+        if (s < t0 * k) atomicAdd(&cnt_before[e], 1);
+        else if (s < t1 * k) my_ids[s - t0 * k] = e;
+      }
+    }
   }
   __syncthreads();
   // offsets of the experts; union flags and work-entry counts (every CTA has
