@@ -96,6 +96,13 @@ Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret, int32_
   d.k = top_k;
   d.m_ret = m_ret;
   d.tok_chunk = token_chunk_for(d.B, top_k, m_ret);
+  if (Is > 0) {
+    // the shared expert takes every token: at least 64 of them per entry, so
+    // its weight tiles pass through the SMs B/64 times rather than B/16
+    // (a larger token slot per stage, a few stages fewer for the routed items)
+    const int want = pow2_at_least(d.B) < 64 ? pow2_at_least(d.B) : 64;
+    if (d.tok_chunk < want) d.tok_chunk = want;
+  }
   d.Is = Is;
   d.S = Is > 0 ? (d.B + d.tok_chunk - 1) / d.tok_chunk : 0;
   return d;
