@@ -349,6 +349,14 @@ def test_long_combine_lists_all_outputs(tiny, fill):
     _check_out(out.float().cpu().numpy(), ref["out"])
 
 
+@pytest.mark.parametrize("B", [127, 128])
+def test_combine_queue_threshold(tiny, B):
+    # k = 2 of m' = 8: the grid-wide combine queue is used from B * k = 32 m'
+    # (B = 128) on; one token below it every combine is done by the item that
+    # completes it.  Both sides match the oracle on every output.
+    _case(tiny, B=B, m_prime=8, seed_x=31 + B, seed_imp=6, k=2)
+
+
 def test_duplicate_retained_id_is_reported(tiny):
     shape = tiny.shape
     x = synth.hidden_states(4, shape, 4).to(DEV)
