@@ -58,8 +58,12 @@ __host__ __device__ inline int token_box_for(int n16) {
 constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
 // Tokens per routing cluster.  Up to 4 a routing CTA stages its hidden rows
 // in under 17 KiB of shared memory and fits beside a persistent expert-FFN
-// CTA; with 8 it stages 64 KiB and never does.
-inline int route_tokens_per_cluster(int B) { return B <= 32 ? 1 : B <= 64 ? 2 : B <= 256 ? 4 : 8; }
+// CTA; with 8 or 16 it stages 64 KiB and never does.  Above 304 tokens,
+// clusters of 8 would need a second wave of CTAs (two per SM), so they take
+// 16 tokens, staged as bf16.
+inline int route_tokens_per_cluster(int B) {
+  return B <= 32 ? 1 : B <= 64 ? 2 : B <= 256 ? 4 : B <= 304 ? 8 : 16;
+}
 
 // Control words at the head of the workspace (int32 each).
 enum CtrlWord {

@@ -90,13 +90,17 @@ __device__ __forceinline__ void fma_chunk2(const XT *xs, int H, int col, float4 
 // Hidden rows are staged as fp32 unless that would keep a routing CTA from
 // fitting beside a persistent expert-FFN CTA (about 20 KiB of shared memory
 // are left there): TB = 4 stays bf16; with TB = 8 no routing CTA fits beside
-// one anyway.
+// one anyway.  TB = 16 stays bf16 too, so that two CTAs fit on an SM.
 template <int TB>
 struct StageType {
   using T = float;
 };
 template <>
 struct StageType<4> {
+  using T = __nv_bfloat16;
+};
+template <>
+struct StageType<16> {
   using T = __nv_bfloat16;
 };
 
@@ -449,7 +453,8 @@ cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w
     case 1: return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
     case 2: return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
     case 4: return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);
-    default: return launch_route_nc<8>(hidden, router_w, retained, d, ws, pdl, stream);
+    case 8: return launch_route_nc<8>(hidden, router_w, retained, d, ws, pdl, stream);
+    default: return launch_route_nc<16>(hidden, router_w, retained, d, ws, pdl, stream);
   }
 }
 
