@@ -51,7 +51,7 @@ typedef enum slimwise_status {
 
 /* Device-side error bits reported by slimwise_moe_device_status(). */
 #define SLIMWISE_DEVERR_PIPELINE_TIMEOUT 0x1   /* an mbarrier wait gave up        */
-#define SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT 0x2 /* gate/up -> down wait gave up    */
+#define SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT 0x2 /* gate/up -> down, or combine-queue, wait gave up */
 #define SLIMWISE_DEVERR_DUPLICATE_RETAINED 0x4 /* retained_idx has a repeated id  */
 #define SLIMWISE_DEVERR_BAD_RETAINED 0x8       /* retained_idx has an id outside [0,E) */
 #define SLIMWISE_DEVERR_BAD_TOPK 0x10          /* a given top-k id outside [0,E)  */
