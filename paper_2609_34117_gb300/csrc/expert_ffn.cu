@@ -30,6 +30,9 @@
 //            entry's tokens (after all its gate/up tiles are done); epilogue
 //            stores fp32 y; the last of the k contributions to a
 //            (token, h-tile) sums sum_j g[t,j] y_j in j order and writes bf16.
+//            At 32 or more tokens per retained expert it combines 8 of its
+//            tokens itself and queues the rest in the workspace; epilogue
+//            groups with no items left drain that queue.
 // Every wait is bounded (1 s): on timeout the CTA records an error bit in the
 // workspace, stops taking work, drains its own copies and MMAs, frees TMEM
 // and exits.
