@@ -483,8 +483,10 @@ def main_gpu(args, ws, rank, local):
     shape = SHAPES[wl.get("shape", "qwen")]
     B, m_prime = wl["B"], wl["m_prime"]
     # one weight copy is enough when the touched bytes exceed L2 several times;
-    # the sweep rotates 4 copies for its small-batch points
-    copies = 4 if args.sweep else 1
+    # otherwise (the sweep's small points, the most-pruned layers) 4 copies
+    # rotate, as they do wherever the measured union stays under 4 x L2
+    most_touched = min(m_prime, B * shape.top_k) * shape.expert_bytes
+    copies = 4 if (args.sweep or most_touched < 4 * L2_BYTES) else 1
     layer = LayerInputs(shape, seed=0, device=device, copies=copies, shared=wl.get("shared", 0))
     sweep_layer = layer if layer.shared is None else LayerInputs(shape, 0, device, copies)
     if wl.get("compact"):
