@@ -426,6 +426,35 @@ def test_zipf_skewed_layers_route_exactly(qwen):
     assert np.mean(us) < m_prime * (1 - (1 - 8 / m_prime) ** Bs)
 
 
+def test_layer_stack_back_to_back():
+    # three distinct Qwen-class layers (own weights, retained set and Zipf(1.1)
+    # popularity) run back to back through one workspace, as the layers of a
+    # decode step's MoE stack do; each layer's routing is checked exactly and
+    # its outputs on a sample of tokens
+    shape = synth.QWEN
+    B, m_prime, k = 256, 64, shape.top_k
+    x0 = synth.hidden_states(B, shape, 41)
+    ws = sw.alloc_workspace(B, shape.hidden, shape.num_experts, shape.inter, k, DEV)
+    runs = []
+    for l in range(3):
+        layer = Layer(shape, seed=5000 + l)
+        bias = synth.zipf_rank_bias(shape.num_experts, 1.1, 9000 + l)
+        x, wr = synth.apply_popularity_bias(x0, layer.wr, bias)
+        ret = synth.retained_set(shape.num_experts, m_prime, 7000 + l)
+        out = sw.slimwise_moe_decode(x.to(DEV), wr.to(DEV), ret.to(DEV), layer.d_w_gu,
+                                     layer.d_w_d, k, workspace=ws)
+        runs.append((layer, x, wr, ret, out))
+    torch.cuda.synchronize()
+    assert sw.slimwise_moe_device_status(ws) == 0
+    tokens = np.sort(np.random.default_rng(3).choice(B, size=4, replace=False)).astype(np.int32)
+    for layer, x, wr, ret, out in runs:
+        route = sw.slimwise_moe_route(x.to(DEV), wr.to(DEV), ret.to(DEV), k, shape.num_experts,
+                                      shape.inter)
+        ref = _oracle(layer, x, ret, k, tokens=tokens, wr=wr)
+        _check_route({n: t.cpu().numpy() for n, t in route.items()}, ref, shape.num_experts)
+        _check_out(out.float().cpu().numpy()[tokens], ref["out"])
+
+
 # --------------------------------------------------------------------------
 # Expert-importance statistics and the retained set (Sec. 2.3, Sec. 3.1)
 # --------------------------------------------------------------------------
