@@ -227,7 +227,7 @@ template <bool kShared>
 __global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
-                      int tmem_cols) {
+                      int tmem_cols, int static_first) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -345,8 +345,15 @@ __global__ void __maxnreg__(128)
       int slot = 0;
       uint32_t rphase = 0;
       int issued = 0;
+      // With every CTA of the grid resident (one per SM), CTA i's first item
+      // is item i and later ones come from the counter past the grid: the
+      // first item costs no atomic round trip after the dependency wait.
+      bool first = static_first != 0;
       for (;;) {
-        int item = atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
+        int item = first ? (int)blockIdx.x
+                         : (static_first ? (int)gridDim.x : 0) +
+                               atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
+        first = false;
         if (*abort) item = 0x7FFFFFFF;
         if (!mbar_wait_bounded(ite_bar(slot), rphase ^ 1u, abort, kTimeoutNs)) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
@@ -734,8 +741,10 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  int optin = 0;
+  int optin = 0, sms = 0;
   err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (err != cudaSuccess) return err;
+  err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (err != cudaSuccess) return err;
   // the token maps exist for boxes of 16 << m <= tok_chunk rows, and an
   // entry's box covers at most tok_chunk rows: tok_chunk must be a power of
@@ -765,7 +774,10 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols);
+  // items are assigned statically to first CTAs only if all of them are
+  // resident at once (a down item may wait on another CTA's first item)
+  const int static_first = grid <= sms ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols, static_first);
 }
 
 }  // namespace slimwise
