@@ -8,7 +8,7 @@ I=768, top-8, decode batch 64 (1.19 GB of touched expert weights per step,
 larger than the 129 MB L2).  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl slimwise|reference]
-                  [--workload qwen_full_b64|qwen_p50_b64|qwen_p50_b128|qwen_p50_b256]
+                  [--workload qwen_full_b64|qwen_p50_b64|... (see WORKLOADS)]
                   [--sweep] [--stack40]
 
 Under torchrun (N > 1) every rank runs an independent replica of the layer on
@@ -45,6 +45,9 @@ WORKLOADS = {
     "qwen_p50_b64": dict(B=64, m_prime=64),
     "qwen_p50_b128": dict(B=128, m_prime=64),
     "qwen_p50_b256": dict(B=256, m_prime=64),
+    # the sweep's largest batch at 75 % pruning: 128 tokens per expert, where
+    # the grid-wide combine queue and 16-token routing clusters are in use
+    "qwen_p75_b512": dict(B=512, m_prime=32),
     # the same 50 % pool as a compact checkpoint holding only the retained
     # experts (full-pool entry point on [m', ...] tensors)
     "qwen_compact_p50_b64": dict(B=64, m_prime=64, compact=True),
@@ -516,8 +519,10 @@ def main_gpu(args, ws, rank, local):
                    "shared_expert_inter": wl.get("shared", 0),
                    "union_mean": pt["union_mean"], "union_eq1": pt["union_eq1"],
                    "parallelism": f"replicas{ws}",
-                   "l2": "touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
-                         % ((pt["union_mean"] * shape.expert_bytes + layer.shared_bytes()) / 1e9)},
+                   "l2": ("touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
+                          % ((pt["union_mean"] * shape.expert_bytes + layer.shared_bytes()) / 1e9)
+                          + ("; %d weight copies rotated across steps" % pt["weight_copies_rotated"]
+                             if pt["weight_copies_rotated"] > 1 else ""))},
         "touched_hbm": {"gbs": pt["touched_gbs"], "frac_of_8tbs": pt["touched_gbs"] / NOMINAL_HBM_GBS,
                         "frac_of_measured": pt["touched_gbs"] / peak},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
