@@ -174,9 +174,9 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   const int nt = min(TB, d.B - t0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // Retained ids, clamped into [0, E) so a bad id cannot fault; the last CTA
-  // (off the critical path of cluster 0's top-k) reports bad and repeated ids
-  // and resets the error word of this call.
+  // Retained ids, clamped into [0, E) so a bad id cannot fault; the grid's
+  // last CTA also reports bad and repeated ids and resets the error word of
+  // this call.
   for (int r = threadIdx.x; r < m; r += blockDim.x) {
     int e = retained ? retained[r] : r;
     ids[r] = min(max(e, 0), d.E - 1);
