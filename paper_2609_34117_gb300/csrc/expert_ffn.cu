@@ -335,6 +335,10 @@ __global__ void __maxnreg__(128)
   ip.S = kShared ? d.S : 0;
   const int nb_cols = d.tok_chunk;  // TMEM columns per accumulator buffer
 
+  const int total_down = total - ip.r1 - ip.S * ip.t1s;  // down items of the launch
+  const int q_cap = d.B * t2;                            // combine-queue slots
+  const bool comb_queue = use_combine_queue(d);
+
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
@@ -541,9 +545,6 @@ __global__ void __maxnreg__(128)
     int *q_base = gm + 1;
     int *comb_list = gm + 2;                          // [kMaxTokTile]
     const int ew = q;                                 // warp within the group
-    const int total_down = total - ip.r1 - ip.S * ip.t1s;  // down items of the launch
-    const int q_cap = d.B * t2;                            // combine-queue slots
-    const bool comb_queue = use_combine_queue(d);
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
@@ -679,35 +680,37 @@ __global__ void __maxnreg__(128)
         }
       }
     }
-    // No items left for this group: take queued combines, each warp one slot
-    // at a time, until it draws a closed slot.
-    while (comb_queue && !*abort && total_down > 0) {
-      int v = -1;
-      if (lane == 0) {
-        const int h = atomicAdd(&ws.ctrl[kCtrlCombHead], 1);
-        if (h < q_cap) {
-          const uint64_t t0 = global_timer_ns();
-          uint32_t nap = 64;
-          for (;;) {
-            const int x = ld_acquire(&ws.comb_q[h]);
-            if (x != 0) {
-              v = x;
-              break;
-            }
-            if (*abort) break;
-            if (global_timer_ns() - t0 > kTimeoutNs) {
-              raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
-              break;
-            }
-            __nanosleep(nap);
-            if (nap < 1024) nap <<= 1;
+  }
+
+  // Every warp with no work left (producer, MMA issuer and the epilogue
+  // groups) takes queued combines, one slot at a time, until it draws a
+  // closed slot.
+  while (comb_queue && !*abort && total_down > 0) {
+    int v = -1;
+    if (lane == 0) {
+      const int h = atomicAdd(&ws.ctrl[kCtrlCombHead], 1);
+      if (h < q_cap) {
+        const uint64_t t0 = global_timer_ns();
+        uint32_t nap = 64;
+        for (;;) {
+          const int x = ld_acquire(&ws.comb_q[h]);
+          if (x != 0) {
+            v = x;
+            break;
           }
+          if (*abort) break;
+          if (global_timer_ns() - t0 > kTimeoutNs) {
+            raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
+            break;
+          }
+          __nanosleep(nap);
+          if (nap < 1024) nap <<= 1;
         }
       }
-      v = __shfl_sync(0xFFFFFFFFu, v, 0);
-      if (v <= 0 || v > q_cap) break;
-      combine_token<kShared>(ws, d, out, (v - 1) / t2, (v - 1) % t2, lane);
     }
+    v = __shfl_sync(0xFFFFFFFFu, v, 0);
+    if (v <= 0 || v > q_cap) break;
+    combine_token<kShared>(ws, d, out, (v - 1) / t2, (v - 1) % t2, lane);
   }
 
   tc_fence_before();
