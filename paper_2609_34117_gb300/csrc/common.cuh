@@ -58,11 +58,17 @@ __host__ __device__ inline int token_box_for(int n16) {
 constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
 // Tokens per routing cluster.  Up to 4 a routing CTA stages its hidden rows
 // in under 17 KiB of shared memory and fits beside a persistent expert-FFN
-// CTA; with 8 or 16 it stages 64 KiB and never does.  Above 304 tokens,
-// clusters of 8 would need a second wave of CTAs (two per SM), so they take
-// 16 tokens, staged as bf16.
-inline int route_tokens_per_cluster(int B) {
-  return B <= 32 ? 1 : B <= 64 ? 2 : B <= 256 ? 4 : B <= 304 ? 8 : 16;
+// CTA; with 8 or 16 it stages 64 KiB and never does.  One wave of routing
+// CTAs (two per SM) holds 38 clusters: above 152 tokens clusters of 4 need
+// two waves, so pools of at most 64 retained experts (small slices per CTA)
+// take 8 tokens per cluster there; above 304 tokens every pool takes 16,
+// staged as bf16.
+inline int route_tokens_per_cluster(int B, int m_ret) {
+  if (B <= 32) return 1;
+  if (B <= 64) return 2;
+  if (B <= 152) return 4;
+  if (B <= 256) return m_ret <= 64 ? 8 : 4;
+  return B <= 304 ? 8 : 16;
 }
 
 // Control words at the head of the workspace (int32 each).

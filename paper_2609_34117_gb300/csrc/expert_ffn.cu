@@ -757,7 +757,7 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   // leave room on each SM for the next layer's routing CTAs, which become
   // resident while this grid finishes (programmatic dependent launch), where
   // they can fit at all: routing CTAs of 8 tokens never do
-  const size_t reserve = route_tokens_per_cluster(d.B) <= 4 ? kCoResidentSmem : 0;
+  const size_t reserve = route_tokens_per_cluster(d.B, d.m_ret) <= 4 ? kCoResidentSmem : 0;
   const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - reserve);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;

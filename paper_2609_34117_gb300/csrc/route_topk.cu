@@ -449,7 +449,7 @@ cudaError_t launch_route_nc(const __nv_bfloat16 *hidden, const float *router_w,
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
                               const int32_t *retained, Dims d, Ws ws, bool pdl,
                               cudaStream_t stream) {
-  switch (route_tokens_per_cluster(d.B)) {
+  switch (route_tokens_per_cluster(d.B, d.m_ret)) {
     case 1: return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
     case 2: return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
     case 4: return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);
