@@ -279,6 +279,19 @@ def test_top_k_extremes(tiny, k):
     _case(tiny, B=12, m_prime=8, seed_x=7, seed_imp=3, k=k)
 
 
+@pytest.mark.parametrize("B,k", [(33, 12), (300, 16)])
+def test_top_k_above_8(tiny, B, k):
+    # the full tiny pool (16 experts) with k > 8: every combine sums two
+    # batches of selections, and at B = 300 (k * B >= 32 m') the combine
+    # queue is in use
+    _case(tiny, B=B, m_prime=None, seed_x=50 + k, seed_imp=0, k=k)
+
+
+def test_top_k_32_qwen(qwen):
+    # the largest k the ABI accepts, on the Qwen-class full pool
+    _case(qwen, B=8, m_prime=None, seed_x=61, seed_imp=0, k=32, sample=4)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
