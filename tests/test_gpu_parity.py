@@ -292,6 +292,15 @@ def test_top_k_32_qwen(qwen):
     _case(qwen, B=8, m_prime=None, seed_x=61, seed_imp=0, k=32, sample=4)
 
 
+@pytest.mark.parametrize("B", [37, 200])
+def test_generic_shape(B):
+    # H = 640 (five 128-wide chunks: ragged batches of router-row loads, five
+    # combine tiles), I = 192 (three gate/up tiles), 24 experts, top-3 of 12;
+    # B = 200 puts the combine queue in use
+    layer = Layer(synth.LayerShape(hidden=640, num_experts=24, inter=192, top_k=3), seed=3)
+    _case(layer, B=B, m_prime=12, seed_x=70 + B, seed_imp=4)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
