@@ -301,6 +301,15 @@ def test_generic_shape(B):
     _case(layer, B=B, m_prime=12, seed_x=70 + B, seed_imp=4)
 
 
+@pytest.mark.parametrize("B", [5, 90])
+def test_generic_shape_with_shared_expert(B):
+    # the generic shape with a shared expert of width 192 (three gate/up
+    # tiles, three down K stages); B = 90 makes two shared entries of 64
+    layer = Layer(synth.LayerShape(hidden=640, num_experts=24, inter=192, top_k=3), seed=3)
+    se = SharedExpert(layer, 192, seed=33)
+    _case_shared(layer, se, B=B, m_prime=12, seed_x=80 + B, seed_imp=4)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
