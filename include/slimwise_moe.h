@@ -56,7 +56,9 @@ typedef enum slimwise_status {
 #define SLIMWISE_DEVERR_BAD_RETAINED 0x8       /* retained_idx has an id outside [0,E) */
 #define SLIMWISE_DEVERR_BAD_TOPK 0x10          /* a given top-k id outside [0,E)  */
 
-/* Problem shape. */
+/* Problem shape.  Supported: 0 <= B <= 2^20; H a multiple of 128 in
+ * [128, 32768]; I a multiple of 64 in [64, 65536]; 1 <= E <= 1024.  Others
+ * return SLIMWISE_ERR_UNSUPPORTED_SHAPE (B out of range: INVALID_ARG). */
 typedef struct slimwise_moe_shape {
   int32_t num_tokens;  /* B: decode batch (tokens)           */
   int32_t hidden;      /* H: model width                     */

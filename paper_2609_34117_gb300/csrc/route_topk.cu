@@ -410,13 +410,18 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
 #endif
 }
 
+// Dynamic shared memory of a routing CTA with TB tokens.
+template <int TB>
+size_t route_smem_bytes(const Dims &d) {
+  return (size_t)TB * d.H * sizeof(typename StageType<TB>::T) +
+         (size_t)((TB + kClusterCtas - 1) / kClusterCtas) * d.m_ret * 4 + (size_t)d.m_ret * 4;
+}
+
 template <int TB, int NC>
 cudaError_t launch_route_tb(const __nv_bfloat16 *hidden, const float *router_w,
                             const int32_t *retained, Dims d, Ws ws, bool pdl,
                             cudaStream_t stream) {
-  const size_t smem = (size_t)TB * d.H * sizeof(typename StageType<TB>::T) +
-                      (size_t)((TB + kClusterCtas - 1) / kClusterCtas) * d.m_ret * 4 +
-                      (size_t)d.m_ret * 4;
+  const size_t smem = route_smem_bytes<TB>(d);
   cudaError_t err = cudaFuncSetAttribute(
       route_topk_kernel<TB, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
@@ -449,7 +454,21 @@ cudaError_t launch_route_nc(const __nv_bfloat16 *hidden, const float *router_w,
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
                               const int32_t *retained, Dims d, Ws ws, bool pdl,
                               cudaStream_t stream) {
-  switch (route_tokens_per_cluster(d.B, d.m_ret)) {
+  int dev = 0, optin = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (err != cudaSuccess) return err;
+  // wide hidden rows: fewer tokens per cluster until they fit in shared memory
+  int tb = route_tokens_per_cluster(d.B, d.m_ret);
+  auto fits = [&](int t) {
+    const size_t need = t == 16 ? route_smem_bytes<16>(d) : t == 8 ? route_smem_bytes<8>(d)
+                      : t == 4 ? route_smem_bytes<4>(d) : t == 2 ? route_smem_bytes<2>(d)
+                      : route_smem_bytes<1>(d);
+    return need <= (size_t)optin;
+  };
+  while (tb > 1 && !fits(tb)) tb >>= 1;
+  switch (tb) {
     case 1: return launch_route_nc<1>(hidden, router_w, retained, d, ws, pdl, stream);
     case 2: return launch_route_nc<2>(hidden, router_w, retained, d, ws, pdl, stream);
     case 4: return launch_route_nc<4>(hidden, router_w, retained, d, ws, pdl, stream);

@@ -73,7 +73,8 @@ bool aligned(const void *p, uintptr_t a) {
 int check_shape(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret) {
   if (!s) return SLIMWISE_ERR_INVALID_ARG;
   if (s->num_tokens < 0 || s->num_tokens > (1 << 20)) return SLIMWISE_ERR_INVALID_ARG;
-  if (s->hidden < 128 || s->hidden % 128 != 0 || s->hidden > 65536)
+  // a routing CTA stages at least one fp32 hidden row in shared memory
+  if (s->hidden < 128 || s->hidden % 128 != 0 || s->hidden > 32768)
     return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
   if (s->inter < 64 || s->inter % 64 != 0 || s->inter > 65536)
     return SLIMWISE_ERR_UNSUPPORTED_SHAPE;

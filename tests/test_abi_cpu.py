@@ -56,6 +56,7 @@ def test_workspace_size_grows_with_batch_and_covers_buffers(lib):
 
 @pytest.mark.parametrize("B,H,E,I,k,code", [
     (4, 100, 16, 128, 2, 2),     # H not a multiple of 128
+    (4, 32896, 16, 128, 2, 2),   # H above 32768
     (4, 256, 16, 96, 2, 2),      # I not a multiple of 64
     (4, 256, 2000, 128, 2, 2),   # too many experts
     (4, 256, 16, 128, 0, 1),     # top_k = 0

@@ -310,6 +310,14 @@ def test_generic_shape_with_shared_expert(B):
     _case_shared(layer, se, B=B, m_prime=12, seed_x=80 + B, seed_imp=4)
 
 
+@pytest.mark.parametrize("B", [200, 400])
+def test_wide_hidden(B):
+    # H = 8192: 8 or 16 tokens per routing cluster would stage more hidden
+    # rows than a CTA's shared memory holds, so the clusters take fewer tokens
+    layer = Layer(synth.LayerShape(hidden=8192, num_experts=64, inter=128, top_k=4), seed=5)
+    _case(layer, B=B, m_prime=32, seed_x=90 + B, seed_imp=6, sample=4)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
