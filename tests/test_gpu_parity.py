@@ -318,6 +318,14 @@ def test_wide_hidden(B):
     _case(layer, B=B, m_prime=32, seed_x=90 + B, seed_imp=6, sample=4)
 
 
+@pytest.mark.parametrize("E,m_prime,k,B", [(512, 384, 8, 40), (1024, 1024, 32, 4)])
+def test_large_pools(E, m_prime, k, B):
+    # more than 256 retained experts: the routing's general top-k (candidates
+    # in a local array), up to the largest pool and k the ABI accepts
+    layer = Layer(synth.LayerShape(hidden=256, num_experts=E, inter=64, top_k=k), seed=7)
+    _case(layer, B=B, m_prime=None if m_prime == E else m_prime, seed_x=95 + B, seed_imp=8)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
