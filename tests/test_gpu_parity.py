@@ -326,6 +326,12 @@ def test_large_pools(E, m_prime, k, B):
     _case(layer, B=B, m_prime=None if m_prime == E else m_prime, seed_x=95 + B, seed_imp=8)
 
 
+def test_wide_intermediate():
+    # I = 4096: 64 gate/up tiles per entry and 64 K stages per down item
+    layer = Layer(synth.LayerShape(hidden=256, num_experts=8, inter=4096, top_k=2), seed=9)
+    _case(layer, B=10, m_prime=6, seed_x=97, seed_imp=10)
+
+
 def test_zero_tokens_is_noop(tiny):
     x = torch.empty((0, tiny.shape.hidden), dtype=torch.bfloat16, device=DEV)
     out = sw.slimwise_moe_decode_full(x, tiny.d_wr, tiny.d_w_gu, tiny.d_w_d, 2)
