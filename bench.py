@@ -300,8 +300,9 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     t1.record(stream)
     torch.cuda.synchronize()
     step_ms = t0.elapsed_time(t1) / steps
-    # expert-FFN kernel alone, events on the launch stream
-    ksteps = min(steps, 400)
+    # expert-FFN kernel alone, events on the launch stream (at least 400
+    # launches whatever K is, so the clock sampler sees the GPU under load)
+    ksteps = max(400, min(steps, 1000))
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(ksteps)]
     for a, b in evs:   # torch creates the CUDA event on its first record
         a.record(stream)
@@ -313,7 +314,7 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     # spread: events around blocks of 10 consecutive layer calls (an event
     # between every two calls would block the programmatic launch overlap)
     block = 10
-    nblocks = max(10, min(steps // block, 100))
+    nblocks = max(40, min(steps // block, 100))
     marks = [torch.cuda.Event(enable_timing=True) for _ in range(nblocks + 1)]
     for ev in marks:
         ev.record(stream)
@@ -474,6 +475,45 @@ def cpu_baseline(layer, B, m_prime, budget_s=15.0):
             "host_cpus": os.cpu_count()}
 
 
+def weight_copies(wl, shape, sweep=False):
+    """Weight copies a workload rotates through: one when the most expert bytes
+    a step can touch exceed L2 several times, otherwise four."""
+    B, m_prime = wl["B"], wl["m_prime"]
+    most_touched = min(m_prime, B * shape.top_k) * shape.expert_bytes
+    return 4 if (sweep or most_touched < 4 * L2_BYTES) else 1
+
+
+def eq1_union(B, m_prime, k):
+    """Expected distinct experts of a batch under uniform routing (Eq. 1)."""
+    return m_prime * (1 - (1 - k / m_prime) ** B)
+
+
+def workload_rotation(wl, shape):
+    """Weight copies the GPU arm rotates across steps for this workload: four
+    when the expected touched bytes (Eq. 1 union) stay under 4 x L2, else one."""
+    touched = eq1_union(wl["B"], wl["m_prime"], shape.top_k) * shape.expert_bytes
+    touched += 6 * shape.hidden * wl.get("shared", 0)
+    copies = weight_copies(wl, shape)
+    return copies if (copies > 1 and touched < 4 * L2_BYTES) else 1
+
+
+def workload_config(name, wl, shape, ws):
+    """The `config` object of a bench line.  It depends on the workload alone,
+    so both arms print the same object; measured unions go in 'union'."""
+    B, m_prime, k = wl["B"], wl["m_prime"], shape.top_k
+    touched = eq1_union(B, m_prime, k) * shape.expert_bytes + 6 * shape.hidden * wl.get("shared", 0)
+    l2 = ("touched expert weights about %.2f GB per step (Eq. 1 union) > 129 MB L2 (no flush needed)"
+          % (touched / 1e9))
+    rotated = workload_rotation(wl, shape)
+    if rotated > 1:
+        l2 += "; %d weight copies rotated across steps" % rotated
+    return {"workload": name, "hidden": shape.hidden, "experts": shape.num_experts,
+            "retained": m_prime, "inter": shape.inter, "top_k": k, "batch": B,
+            "form": "compact checkpoint" if wl.get("compact") else "masked pool",
+            "shared_expert_inter": wl.get("shared", 0),
+            "parallelism": f"replicas{ws}", "l2": l2}
+
+
 def main_gpu(args, ws, rank, local):
     import paper_2609_34117_gb300 as sw
     from paper_2609_34117_gb300 import build as swbuild
@@ -488,10 +528,10 @@ def main_gpu(args, ws, rank, local):
     # one weight copy is enough when the touched bytes exceed L2 several times;
     # otherwise (the sweep's small points, the most-pruned layers) 4 copies
     # rotate, as they do wherever the measured union stays under 4 x L2
-    most_touched = min(m_prime, B * shape.top_k) * shape.expert_bytes
-    copies = 4 if (args.sweep or most_touched < 4 * L2_BYTES) else 1
+    copies = weight_copies(wl, shape, args.sweep)
     layer = LayerInputs(shape, seed=0, device=device, copies=copies, shared=wl.get("shared", 0))
     sweep_layer = layer if layer.shared is None else LayerInputs(shape, 0, device, copies)
+    full_shape = shape
     if wl.get("compact"):
         layer = layer.compacted(m_prime)
         shape = layer.shape
@@ -513,16 +553,9 @@ def main_gpu(args, ws, rank, local):
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": pt["step_ms"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
-                   "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B,
-                   "form": "compact checkpoint" if wl.get("compact") else "masked pool",
-                   "shared_expert_inter": wl.get("shared", 0),
-                   "union_mean": pt["union_mean"], "union_eq1": pt["union_eq1"],
-                   "parallelism": f"replicas{ws}",
-                   "l2": ("touched expert weights %.2f GB per step > 129 MB L2 (no flush needed)"
-                          % ((pt["union_mean"] * shape.expert_bytes + layer.shared_bytes()) / 1e9)
-                          + ("; %d weight copies rotated across steps" % pt["weight_copies_rotated"]
-                             if pt["weight_copies_rotated"] > 1 else ""))},
+        "config": workload_config(args.workload, wl, full_shape, ws),
+        "union": {"mean": pt["union_mean"], "eq1": pt["union_eq1"],
+                  "weight_copies_rotated": pt["weight_copies_rotated"]},
         "touched_hbm": {"gbs": pt["touched_gbs"], "frac_of_8tbs": pt["touched_gbs"] / NOMINAL_HBM_GBS,
                         "frac_of_measured": pt["touched_gbs"] / peak},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -537,8 +570,11 @@ def main_gpu(args, ws, rank, local):
         "gpu_launches": 3 * args.steps,
         "clocks": clk.summary(),
     }
+    if not args.no_pruned:
+        result["pruned"] = run_pruned(sw, device, peak, local)
     if args.sweep:
-        result["sweep"] = run_sweep(sw, sweep_layer, device, peak)
+        result["sweep"] = run_sweep(sw, sweep_layer, device, peak,
+                                    cpu=rank == 0 and not args.no_cpu_baseline)
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(layer, B, m_prime)
     elif rank == 0:
@@ -546,12 +582,63 @@ def main_gpu(args, ws, rank, local):
     if args.stack40:
         del layer
         torch.cuda.empty_cache()
-        result["stack40"] = run_stack40(sw, device, max(3, min(args.steps // 100, 20)), 2, peak)
+        result["stack40"] = run_stack40(sw, device, max(3, min(args.steps // 100, 20)), 2, peak,
+                                        cpu=rank == 0 and not args.no_cpu_baseline)
     if rank == 0:
         print(json.dumps(result), flush=True)
 
 
-def run_stack40(sw, device, steps, warmup, peak, n_layers=40, B=256, m_prime=64):
+PRUNED_POINTS = ("qwen_p50_b64", "qwen_p50_b256", "qwen_p75_b64")
+
+
+def run_pruned(sw, device, peak, local, steps=4000):
+    """The pruned Qwen-class layer at the target's points (50 % pruning at
+    B = 64 and 256, 75 % at B = 64): each point times `steps` layer calls
+    under its own clock sampler.  'touched' is the union's weight bytes over
+    the whole step time (routing + grouping + FFN)."""
+    shape = synth.QWEN
+    layer = LayerInputs(shape, seed=0, device=device, copies=4)
+    pts = []
+    for name in PRUNED_POINTS:
+        wl = WORKLOADS[name]
+        with ClockSampler(local) as clk:
+            p = measure_point(sw, layer, wl["B"], wl["m_prime"], steps, 50, device, seed_x=1)
+        p.pop("_state")
+        pts.append({
+            "workload": name, "batch": wl["B"], "retained": wl["m_prime"], "steps": steps,
+            "union_mean": p["union_mean"], "ms_per_step": p["step_ms"],
+            "tokens_per_s": p["tokens_per_s"], "ffn_ms": p["ffn_ms"],
+            "touched_gbs": p["touched_gbs"],
+            "touched_frac_of_measured": p["touched_gbs"] / peak,
+            "touched_frac_of_8tbs": p["touched_gbs"] / NOMINAL_HBM_GBS,
+            "ffn_frac_of_measured": p["ffn_gbs"] / peak,
+            "step_ms_p10_p50_p90": [p["step_ms_p10"], p["step_ms_p50"], p["step_ms_p90"]],
+            "weight_copies_rotated": p["weight_copies_rotated"],
+            "clocks": clk.summary()})
+    del layer
+    torch.cuda.empty_cache()
+    return pts
+
+
+def cpu_oracle_all_cores(w_gu_bits, w_d_bits, wr, retained, x_bits, k, tokens):
+    """The oracle built with OpenMP over tokens, on all host cores: routing of
+    the whole batch (single thread) and the expert FFNs + combine of `tokens`.
+    Returns (seconds, threads) or None when no OpenMP build is possible."""
+    import oracle
+    try:
+        path = oracle.build_openmp()
+    except (OSError, subprocess.CalledProcessError):
+        return None
+    with oracle.swapped_library(path):
+        threads = oracle.num_threads()
+        t0 = time.perf_counter()
+        idx, gates = oracle.route(oracle.router_logits(x_bits, wr), retained, k)
+        oracle.group_by_expert(idx, wr.shape[0])
+        oracle.experts_combine(x_bits, idx, gates, w_gu_bits, w_d_bits, tokens=tokens)
+        return time.perf_counter() - t0, threads
+
+
+def run_stack40(sw, device, steps, warmup, peak, n_layers=40, B=256, m_prime=64, cpu=False):
     """Decode-step MoE stack: n_layers independent Qwen-class layers (own
     weights, own retained set, own Zipf(1.1) popularity bias), called back to
     back on one stream; one step = all layers over one batch."""
@@ -592,7 +679,28 @@ def run_stack40(sw, device, steps, warmup, peak, n_layers=40, B=256, m_prime=64)
         raise RuntimeError("device error bits set in the stack run")
     ms = t0.elapsed_time(t1) / steps
     touched = sum(us) * shape.expert_bytes
+    cpu_base = None
+    if cpu:
+        # the all-core oracle on the first 3 layers, whole batch each; the
+        # stack's time is their mean per layer times the layer count
+        xb = synth.bf16_bits(x)
+        secs, threads = [], 1
+        for (w_gu, w_d, wr, ret) in layers[:3]:
+            r = cpu_oracle_all_cores(synth.bf16_bits(w_gu), synth.bf16_bits(w_d), wr.cpu().numpy(),
+                                     ret.cpu().numpy(), xb, k, None)
+            if r is None:
+                break
+            secs.append(r[0])
+            threads = r[1]
+        if secs:
+            per_layer = float(np.mean(secs))
+            cpu_base = {"value": B / (per_layer * n_layers), "unit": "tokens/s through the stack",
+                        "cores": threads, "kind": "oracle (OpenMP over tokens)",
+                        "sample": f"layers 0-2 of the {n_layers}, all {B} tokens each "
+                                  f"({sum(secs):.1f} s); stack time = mean per layer x {n_layers}",
+                        "host_cpus": os.cpu_count()}
     return {"layers": n_layers, "B": B, "m_prime": m_prime, "step_ms": ms,
+            "cpu_baseline": cpu_base,
             "tokens_per_s_through_stack": B / (ms * 1e-3),
             "layer_tokens_per_s": B * n_layers / (ms * 1e-3),
             "union_per_layer": us, "union_mean": float(np.mean(us)),
@@ -601,22 +709,42 @@ def run_stack40(sw, device, steps, warmup, peak, n_layers=40, B=256, m_prime=64)
             "weights_gb": n_layers * shape.num_experts * shape.expert_bytes / 1e9}
 
 
-def run_sweep(sw, layer, device, peak):
+def run_sweep(sw, layer, device, peak, cpu=False):
+    gu_bits = dn_bits = wr = None
+    if cpu:
+        w_gu, w_d = layer.copies[0]
+        gu_bits, dn_bits, wr = synth.bf16_bits(w_gu), synth.bf16_bits(w_d), layer.wr.cpu().numpy()
+    shape = layer.shape
     pts = []
     for B in (1, 8, 32, 64, 128, 256, 512):
         for m_prime in (128, 96, 64, 32):
             steps = 300 if B <= 64 else 200
             p = measure_point(sw, layer, B, m_prime, steps, 20, device, seed_x=1000 + B)
-            p.pop("_state")
+            batches, retained = p.pop("_state")[:2]
             p["touched_frac_of_measured"] = p["touched_gbs"] / peak
             p["ffn_frac_of_measured"] = p["ffn_gbs"] / peak
+            if cpu:
+                # the all-core oracle on the point's first batch, every token
+                ret = None if retained is None else retained.cpu().numpy()
+                r = cpu_oracle_all_cores(gu_bits, dn_bits, wr, ret, synth.bf16_bits(batches[0]),
+                                         shape.top_k, None)
+                p["cpu_baseline"] = None if r is None else {
+                    "value": B / r[0], "unit": "tokens/s", "cores": r[1],
+                    "kind": "oracle (OpenMP over tokens)", "sample": f"one batch of {B} tokens",
+                    "host_cpus": os.cpu_count()}
             pts.append(p)
     return pts
 
 
 # ---------------------------------------------------------------- reference arm
 def main_reference(args, ws, rank):
-    """The reference arm is the CPU oracle, timed as it stands on host cores."""
+    """The reference arm is the CPU oracle, timed as it stands on one host core.
+
+    Each step is the layer over one batch: routing of all B tokens, then the
+    expert FFNs and combine of the batch's tokens -- all of them when the
+    whole --steps/--warmup run fits in about two minutes at the oracle's
+    speed, else the first n tokens that fit.  ms_per_step is the measured wall
+    time of a step; value = tokens processed / wall time."""
     if rank != 0:
         return
     import oracle
@@ -632,43 +760,53 @@ def main_reference(args, ws, rank):
     if wl.get("shared"):
         w_sg, gu_s, dn_s = synth.shared_expert(shape.hidden, wl["shared"], 0 + 101)
         se = (w_sg.numpy(), synth.bf16_bits(gu_s), synth.bf16_bits(dn_s))
+    full_shape = shape
     if wl.get("compact"):
         # the retained experts' rows only, in ascending id order
         ids = np.sort(ret)
         gu, dn, wr = np.ascontiguousarray(gu[ids]), np.ascontiguousarray(dn[ids]), np.ascontiguousarray(wr[ids])
         shape = synth.LayerShape(shape.hidden, m_prime, shape.inter, shape.top_k)
         ret = None
-    sample = 4  # tokens whose expert FFNs each step evaluates
+    batches = [synth.bf16_bits(synth.hidden_states(B, shape, 1 + j)) for j in range(N_BATCHES)]
+    # the union of each batch, as the GPU arm reports it
+    unions = [oracle.group_by_expert(oracle.route(oracle.router_logits(xb, wr), ret, shape.top_k)[0],
+                                     shape.num_experts)["union_size"] for xb in batches]
 
-    def step(i):
-        x = synth.bf16_bits(synth.hidden_states(B, shape, 1 + (i % N_BATCHES)))
+    def step(i, n_tok):
+        x = batches[i % N_BATCHES]
         t0 = time.perf_counter()
         z = oracle.router_logits(x, wr)
         idx, gates = oracle.route(z, ret, shape.top_k)
         oracle.group_by_expert(idx, shape.num_experts)
-        t_route = time.perf_counter() - t0
-        toks = [(i * sample + j) % B for j in range(sample)]
-        t1 = time.perf_counter()
+        toks = list(range(n_tok))
         o = oracle.experts_combine(x, idx, gates, gu, dn, tokens=toks)
         if se is not None:
             oracle.shared_expert_add(x, se[0], se[1], se[2], o, tokens=toks)
-        t_ffn = time.perf_counter() - t1
-        return t_route / B + t_ffn / sample   # seconds per token
+        return time.perf_counter() - t0
 
+    # size the step from one timed token so the whole run stays bounded
+    per_tok = step(0, 1)
+    budget_s = 120.0
+    n_tok = int(max(1, min(B, budget_s / (args.steps + args.warmup) / max(per_tok, 1e-6))))
     for i in range(args.warmup):
-        step(i)
-    per_tok = [step(i) for i in range(args.steps)]
-    spt = float(np.mean(per_tok))
-    value = 1.0 / spt
+        step(i, n_tok)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(i, n_tok)
+    wall = time.perf_counter() - t0
+    ms = wall / args.steps * 1e3
+    value = n_tok * args.steps / wall
+    sample = (f"per step: routing of all {B} tokens, expert FFNs + combine of "
+              + (f"all {B} tokens" if n_tok == B else f"the first {n_tok} of {B} tokens")
+              + ", single thread")
     print(json.dumps({
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": spt * B * 1e3, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-        "config": {"workload": args.workload, "hidden": shape.hidden, "experts": shape.num_experts,
-                   "retained": m_prime, "inter": shape.inter, "top_k": shape.top_k, "batch": B},
+        "config": workload_config(args.workload, wl, full_shape, ws),
+        "union": {"mean": float(np.mean(unions)), "eq1": eq1_union(B, m_prime, full_shape.top_k)},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                         "sample": f"per step: routing of all {B} tokens + expert FFNs of {sample} tokens, "
-                                   "single thread, scaled to tokens/s"},
+                         "sample": sample, "host_cpus": os.cpu_count()},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
@@ -684,6 +822,8 @@ def main():
     ap.add_argument("--stack40", action="store_true",
                     help="40 independent skewed layers at m'=64, B=256 (adds 'stack40')")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-pruned", action="store_true",
+                    help="skip the pruned-layer points (adds 'pruned' by default)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -270,15 +270,29 @@ int slimwise_moe_select_retained(const double *stats, int32_t num_experts,
  *   (Qwen-class H=2048, E=128, I=768, top-8: B <= 151); larger problems
  *   return SLIMWISE_ERR_WORKSPACE without launching anything.
  *   The array's device address is looked up on the first call made on each
- *   device; make that first call before any stream capture.
+ *   device; make that first call before any stream capture.  A call that
+ *   returns SLIMWISE_ERR_CUDA drops the cached address, so after a context
+ *   reset (cudaDeviceReset) the next call looks it up again.
  *   All calls share the array: calls whose kernels may overlap on the GPU
  *   (unordered streams) race.  No call allocates or frees memory.
+ *   Device-side errors are read with slimwise_moe_noalloc_device_status().
  */
 int slimwise_moe_decode_noalloc(const void *hidden, const float *router_w,
                                 const int32_t *retained_idx, int32_t n_retained,
                                 const void *w_gate_up, const void *w_down,
                                 int32_t top_k, void *out, void *stream,
                                 const slimwise_moe_shape *shape);
+
+/*
+ * The device error bits (SLIMWISE_DEVERR_*) that the last
+ * slimwise_moe_decode_noalloc call on the current device left in the
+ * library's fixed array, written to *flags after synchronising `stream`.
+ * Returns SLIMWISE_OK if none are set, SLIMWISE_ERR_DEVICE otherwise
+ * (SLIMWISE_ERR_INVALID_ARG for a NULL flags, SLIMWISE_ERR_CUDA if the read
+ * fails).  Like the entry point itself it allocates nothing; the paper has no
+ * counterpart.
+ */
+int slimwise_moe_noalloc_device_status(void *stream, int32_t *flags);
 
 /*
  * Reads (and synchronises `stream` for) the device error bits the last call

@@ -23,6 +23,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "slimwise_oracle.c")
 _BUILD_DIR = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+_OMP_PATH = os.path.join(_BUILD_DIR, "liboracle_omp.so")
 _lock = threading.Lock()
 _lib = None
 
@@ -39,6 +40,26 @@ def build(force: bool = False) -> str:
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
+
+
+def build_openmp(force: bool = False) -> str:
+    """The same source built with -fopenmp: the tokens of the expert/combine
+    step run on all host cores.  Used only to time the oracle on all cores."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if (not force and os.path.exists(_OMP_PATH)
+            and os.path.getmtime(_OMP_PATH) >= os.path.getmtime(_SRC)):
+        return _OMP_PATH
+    tmp = _OMP_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC",
+           "-shared", "-std=c11", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True, capture_output=True)
+    os.replace(tmp, _OMP_PATH)
+    return _OMP_PATH
+
+
+def num_threads() -> int:
+    """Threads the loaded library's token loop uses (1 for the plain build)."""
+    return int(_load().oracle_num_threads())
 
 
 def _load():
@@ -66,6 +87,8 @@ def _load():
             lib.oracle_select_retained.restype = i32
             lib.oracle_moe_decode.argtypes = [P, P, P, i32, P, P, i32, i32, i32, i32, i32, P, P, P]
             lib.oracle_moe_decode.restype = i32
+            lib.oracle_num_threads.argtypes = []
+            lib.oracle_num_threads.restype = i32
             _lib = lib
     return _lib
 
@@ -300,7 +323,8 @@ class swapped_library:
         lib = ctypes.CDLL(self.path)
         for name in ("oracle_router_logits", "oracle_route", "oracle_group_by_expert",
                      "oracle_expert_swiglu", "oracle_experts_combine", "oracle_moe_decode",
-                     "oracle_shared_expert_add", "oracle_expert_stats", "oracle_select_retained"):
+                     "oracle_shared_expert_add", "oracle_expert_stats", "oracle_select_retained",
+                     "oracle_num_threads"):
             fn_new, fn_old = getattr(lib, name), getattr(base, name)
             fn_new.argtypes, fn_new.restype = fn_old.argtypes, fn_old.restype
         with _lock:

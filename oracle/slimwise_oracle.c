@@ -31,12 +31,28 @@
  *     is not rounded.
  *   - the grouping of slots is the stable order (expert asc, token asc).
  *
- * Build: gcc -O2 -ffp-contract=off -fPIC -shared (no fast-math).
+ * Build: gcc -O2 -ffp-contract=off -fPIC -shared (no fast-math).  A second
+ * build with -fopenmp spreads the tokens of oracle_experts_combine over the
+ * host's cores; it is used only to time the oracle on all cores.  Each token
+ * is computed by one thread with the same arithmetic in the same order, so
+ * both builds give identical results.
  */
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Threads the token loop uses: 1 unless built with OpenMP. */
+int oracle_num_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
 
 /* bf16 is the upper half of an fp32 bit pattern. */
 static float bf16_to_float(uint16_t v) {
@@ -211,13 +227,16 @@ int oracle_experts_combine(const uint16_t *x, const int32_t *idx,
                            const double *gates, const uint16_t *w_gate_up,
                            const uint16_t *w_down, int H, int I, int k,
                            const int32_t *tokens, int n_tokens, double *out) {
-  double *a = (double *)malloc(sizeof(double) * (size_t)I);
-  double *y = (double *)malloc(sizeof(double) * (size_t)H);
-  if (!a || !y) {
-    free(a); free(y);
-    return -1;
-  }
+  int failed = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : failed)
   for (int r = 0; r < n_tokens; ++r) {
+    double *a = (double *)malloc(sizeof(double) * (size_t)I);
+    double *y = (double *)malloc(sizeof(double) * (size_t)H);
+    if (!a || !y) {
+      free(a); free(y);
+      failed = 1;
+      continue;
+    }
     int t = tokens[r];
     double *o = out + (size_t)r * H;
     for (int h = 0; h < H; ++h) o[h] = 0.0;
@@ -229,9 +248,9 @@ int oracle_experts_combine(const uint16_t *x, const int32_t *idx,
                            w_down + (size_t)e * H * I, H, I, a, y);
       for (int h = 0; h < H; ++h) o[h] += g * y[h];
     }
+    free(a); free(y);
   }
-  free(a); free(y);
-  return 0;
+  return failed ? -1 : 0;
 }
 
 /*

@@ -34,6 +34,7 @@ EXPORTED = (
     "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
     "slimwise_moe_shared_workspace_size", "slimwise_moe_decode_shared",
     "slimwise_moe_decode_shared_ex", "slimwise_moe_expert_stats", "slimwise_moe_select_retained",
+    "slimwise_moe_noalloc_device_status",
 )
 
 
@@ -79,6 +80,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             lib.slimwise_moe_group.argtypes = [P, i32, P, SP, P, sz] + [P] * 6
             lib.slimwise_moe_device_status.argtypes = [P, P, ctypes.POINTER(i32)]
             lib.slimwise_moe_decode_noalloc.argtypes = [P, P, P, i32, P, P, i32, P, P, SP]
+            lib.slimwise_moe_noalloc_device_status.argtypes = [P, ctypes.POINTER(i32)]
             lib.slimwise_moe_shared_workspace_size.argtypes = [SP, i32, i32, ctypes.POINTER(sz)]
             lib.slimwise_moe_decode_shared.argtypes = [P, P, P, i32, P, P, i32, P, P, P, i32,
                                                        P, P, SP, P, sz]
@@ -359,3 +361,13 @@ def slimwise_moe_decode_noalloc(hidden, router_w, retained_idx, w_gate_up, w_dow
         _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),
         int(top_k), _ptr(out), _stream(stream), ctypes.byref(s)), "slimwise_moe_decode_noalloc")
     return out
+
+
+def slimwise_moe_noalloc_device_status(stream=None) -> int:
+    """Device error bits of the last slimwise_moe_decode_noalloc call on the
+    current device (synchronises the stream)."""
+    flags = ctypes.c_int32(0)
+    rc = load().slimwise_moe_noalloc_device_status(_stream(stream), ctypes.byref(flags))
+    if rc not in (0, 5):
+        _check(rc, "slimwise_moe_noalloc_device_status")
+    return int(flags.value)

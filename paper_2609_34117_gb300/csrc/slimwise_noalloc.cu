@@ -19,6 +19,16 @@
 // there: the kernels set every counter and flag they read at the start of
 // each call, so nothing has to be cleared in between, but two calls whose
 // kernels overlap on the GPU (different streams without ordering) race on it.
+//
+// The kernels record device-side errors (a repeated or out-of-range retained
+// id, a bounded wait that gave up) in the error word at the head of the array;
+// slimwise_moe_noalloc_device_status reads it, as slimwise_moe_device_status
+// does for a caller's workspace.
+//
+// A launch that fails drops the cached address of the current device, so the
+// next call looks it up again: after cudaDeviceReset, or once the primary
+// context was destroyed and created anew, the array may sit at another
+// device address.
 #include <mutex>
 
 #include "common.cuh"
@@ -61,7 +71,25 @@ extern "C" int slimwise_moe_decode_noalloc(const void *hidden, const float *rout
     }
     scratch = g_noalloc_ptr[dev];
   }
-  return slimwise_moe_decode_ex(hidden, router_w, retained_idx, n_retained, w_gate_up,
-                                w_down, top_k, out, stream, shape, scratch,
-                                kNoAllocScratchBytes, nullptr);
+  rc = slimwise_moe_decode_ex(hidden, router_w, retained_idx, n_retained, w_gate_up, w_down,
+                              top_k, out, stream, shape, scratch, kNoAllocScratchBytes, nullptr);
+  if (rc == SLIMWISE_ERR_CUDA) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    g_noalloc_ptr[dev] = nullptr;
+  }
+  return rc;
+}
+
+extern "C" int slimwise_moe_noalloc_device_status(void *stream, int32_t *flags) {
+  if (!flags) return SLIMWISE_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  // the control words are the first region of the scratch layout
+  if (cudaMemcpyFromSymbolAsync(&v, g_noalloc_scratch, sizeof(v),
+                                slimwise::kCtrlErr * sizeof(int32_t), cudaMemcpyDeviceToHost,
+                                st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  *flags = v;
+  return v ? SLIMWISE_ERR_DEVICE : SLIMWISE_OK;
 }

@@ -5,6 +5,7 @@ import os
 import shutil
 import subprocess
 import sys
+import time
 
 import bench
 
@@ -12,10 +13,12 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_reference_arm_prints_one_contract_line():
-    # one timed step of the oracle on this host (a few seconds)
+    # one timed step of the oracle on this host (the whole batch: seconds)
+    t0 = time.perf_counter()
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
                         "--steps", "1", "--warmup", "3"],
                        capture_output=True, text=True, timeout=600, cwd=ROOT)
+    wall = time.perf_counter() - t0
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.strip()]
     assert len(lines) == 1
@@ -26,6 +29,12 @@ def test_reference_arm_prints_one_contract_line():
     assert d["impl"] == "reference" and d["steps"] == 1 and d["warmup"] == 3
     assert d["unit"] == "tokens/s" and d["higher_is_better"] is True and d["value"] > 0
     assert d["config"]["workload"] == "qwen_full_b64"
+    # the same config keys as the GPU arm, and a step time that is measured:
+    # the timed steps fit inside the run's own wall time
+    wl = bench.WORKLOADS["qwen_full_b64"]
+    assert d["config"] == bench.workload_config("qwen_full_b64", wl, bench.synth.QWEN, 1)
+    assert d["config"]["batch"] == 64 and 100 < d["union"]["mean"] <= 128
+    assert d["steps"] * d["ms_per_step"] * 1e-3 < wall
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1
     assert isinstance(cb["sample"], str) and cb["sample"]

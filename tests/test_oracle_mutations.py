@@ -42,6 +42,11 @@ MUTATIONS = {
                            "if (!taken[e] && (best < 0 || score[e] >= score[best])) best = e;"),
     # grouping: offsets off by one expert
     "offsets_shift": ("offsets[e + 1] = offsets[e] + counts[e];", "offsets[e + 1] = offsets[e] + counts[e > 0 ? e - 1 : 0];"),
+    # combine for a token subset: row r computed for token r instead of tokens[r]
+    "combine_token_index": ("    int t = tokens[r];\n    double *o = out + (size_t)r * H;",
+                            "    int t = r;\n    double *o = out + (size_t)r * H;"),
+    # shared expert for a token subset: the same slip
+    "shared_token_index": ("    int t = tokens[r];\n    float z;", "    int t = r;\n    float z;"),
     # grouping: token order reversed inside an expert
     "perm_token_desc": ("for (int t = 0; t < B; ++t)\n    for (int j = 0; j < k; ++j) {\n      int s = t * k + j;",
                         "for (int t = B - 1; t >= 0; --t)\n    for (int j = 0; j < k; ++j) {\n      int s = t * k + j;"),
@@ -62,6 +67,7 @@ PIN_FUNCS = [
     (pins.test_shared_expert_twice_width_is_sum_of_halves, ()),
     (pins.test_expert_stats_totals_and_one_hot_router, ()),
     (pins.test_select_retained_matches_brute_force_with_ties, (0,)),
+    (pins.test_token_subset_rows_equal_whole_batch_rows, ()),
 ]
 
 

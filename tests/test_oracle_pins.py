@@ -235,6 +235,38 @@ def test_golden_fixture_reproduced(oracle_lib):
 
 
 # --------------------------------------------------------------------------
+# Token subsets: the layer is a per-token gate-weighted sum (Sec. 3.1), so the
+# layer evaluated for a subset of the batch gives exactly those tokens' rows
+# --------------------------------------------------------------------------
+def test_token_subset_rows_equal_whole_batch_rows(oracle_lib):
+    shape = synth.TINY
+    x, wr, w_gu, w_d = _tiny_layer(B=9)
+    retained = synth.retained_set(shape.num_experts, 8, seed=2).numpy()
+    xb, w, gu, dn = _bits(x), wr.numpy(), _bits(w_gu), _bits(w_d)
+    k = shape.top_k
+    whole = oracle_lib.moe_decode(xb, w, retained, gu, dn, k)
+    T = np.array([7, 2, 5, 0, 8], np.int32)          # unsorted, not contiguous
+    part = oracle_lib.moe_decode_sampled(xb, w, retained, gu, dn, k, T)
+    assert np.array_equal(part["idx"], whole["idx"])
+    assert np.array_equal(part["out"], whole["out"][T])
+    # each sampled row against a float64 numpy evaluation of its own token
+    x64 = _bf16_to_f64(xb)
+    for r, t in enumerate(T):
+        ref = sum(part["gates"][t, j] * _dense_swiglu(x64[t], _bf16_to_f64(gu[e]), _bf16_to_f64(dn[e]))
+                  for j, e in enumerate(part["idx"][t]))
+        np.testing.assert_allclose(part["out"][r], ref, rtol=1e-10, atol=1e-13)
+    # with the shared expert (Sec. 3.3) each row also carries its own token's
+    # gate and shared term
+    se_gu, se_dn, w_sg = _shared_expert(5, 64)
+    whole_s = oracle_lib.moe_decode_shared(xb, w, retained, gu, dn, k, w_sg, se_gu, se_dn)
+    part_s = oracle_lib.moe_decode_shared(xb, w, retained, gu, dn, k, w_sg, se_gu, se_dn, tokens=T)
+    assert np.array_equal(part_s["shared_gate"], whole_s["shared_gate"][T])
+    assert np.array_equal(part_s["out"], whole_s["out"][T])
+    s_ref = 1.0 / (1.0 + np.exp(-(x64[T] @ w_sg.astype(np.float64))))
+    np.testing.assert_allclose(part_s["shared_gate"], s_ref, rtol=1e-5)
+
+
+# --------------------------------------------------------------------------
 # Batch-permutation invariance
 # --------------------------------------------------------------------------
 def test_batch_permutation_invariance(oracle_lib):
@@ -416,6 +448,33 @@ def test_expert_stats_totals_and_one_hot_router(oracle_lib):
     assert np.all(st0[:k, 0] == 12) and np.all(st0[k:] == 0)
     np.testing.assert_allclose(st0[:k, 1], 12 / k, rtol=1e-14)
     np.testing.assert_allclose(st0[:k, 3], st0[:k, 2] / k, rtol=1e-13)
+
+
+def test_routing_mass_takes_gates_of_selected_experts_only(oracle_lib):
+    # Sec. 2.3 says routing mass aggregates gate probabilities.  The reading
+    # here sums each token's renormalised gates over its k selections, the
+    # weights the layer actually applies (the same gates REAP multiplies the
+    # output norms by).  Summing the pool softmax over every token instead
+    # would credit experts that are never selected: here expert 9 is every
+    # token's runner-up at top-1, with a pool probability near one half and
+    # a routing mass of exactly zero, so the two readings keep different sets.
+    shape = synth.TINY
+    E, B = shape.num_experts, 10
+    x, _, w_gu, w_d = _tiny_layer(B=B)
+    bias = torch.full((E,), -5.0)
+    bias[0], bias[9] = 1.0, 0.99
+    x, wr = synth.apply_popularity_bias(x, torch.zeros((E, shape.hidden)), bias)
+    xb, w, gu, dn = _bits(x), wr.numpy(), _bits(w_gu), _bits(w_d)
+    st = oracle_lib.expert_stats(xb, w, gu, dn, 1)
+    assert st[0, 0] == B and st[0, 1] == B
+    assert np.all(st[1:] == 0)
+    z = oracle_lib.router_logits(xb, w).astype(np.float64)
+    p = np.exp(z - z.max(1, keepdims=True))
+    p /= p.sum(1, keepdims=True)
+    pool_mass = p.sum(0)
+    assert pool_mass[9] > 0.45 * B
+    assert list(oracle_lib.select_retained(st, 2, "mass")) == [0, 1]        # ties to the lowest id
+    assert sorted(np.argsort(-pool_mass, kind="stable")[:2].tolist()) == [0, 9]
 
 
 @pytest.mark.parametrize("seed", [0, 1])
