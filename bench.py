@@ -45,6 +45,7 @@ WORKLOADS = {
     "qwen_p50_b64": dict(B=64, m_prime=64),
     "qwen_p50_b128": dict(B=128, m_prime=64),
     "qwen_p50_b256": dict(B=256, m_prime=64),
+    "qwen_p75_b64": dict(B=64, m_prime=32),
     # the sweep's largest batch at 75 % pruning: 128 tokens per expert, where
     # the grid-wide combine queue and 16-token routing clusters are in use
     "qwen_p75_b512": dict(B=512, m_prime=32),

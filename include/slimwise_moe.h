@@ -123,12 +123,24 @@ int slimwise_moe_decode_full(const void *hidden, const float *router_w,
  *                        ordering instead of programmatic dependent launch.
  *   grid_ctas            >0: persistent expert-FFN grid size (default: the
  *                        device's SM count).
+ *   wait_limit_ns        >0: limit, in ns, of every bounded wait of the
+ *                        expert-FFN kernel (default 1 s).  A wait that runs
+ *                        out sets SLIMWISE_DEVERR_PIPELINE_TIMEOUT or
+ *                        SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT; its CTA then
+ *                        drains its copies and MMAs, frees its tensor memory
+ *                        and exits, and the output is incomplete.
+ *   test_starve_first_down  tests only: 1 makes the first routed down item
+ *                        wait for one more gate/up tile than exists, so that
+ *                        wait runs out after wait_limit_ns (the timeout path).
  */
 typedef struct slimwise_decode_opts {
   void *ffn_begin;
   void *ffn_end;
   int32_t disable_pdl;
   int32_t grid_ctas;
+  int64_t wait_limit_ns;
+  int32_t test_starve_first_down;
+  int32_t reserved;
 } slimwise_decode_opts;
 
 /* slimwise_moe_decode with launch options; retained_idx NULL = full pool. */

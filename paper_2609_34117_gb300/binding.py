@@ -51,7 +51,9 @@ class Shape(ctypes.Structure):
 
 class DecodeOpts(ctypes.Structure):
     _fields_ = [("ffn_begin", ctypes.c_void_p), ("ffn_end", ctypes.c_void_p),
-                ("disable_pdl", ctypes.c_int32), ("grid_ctas", ctypes.c_int32)]
+                ("disable_pdl", ctypes.c_int32), ("grid_ctas", ctypes.c_int32),
+                ("wait_limit_ns", ctypes.c_int64), ("test_starve_first_down", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 def library_path() -> str:
@@ -256,8 +258,9 @@ def slimwise_moe_select_retained(stats, n_retained, criterion="reap", stream=Non
     return ids
 
 
-def _opts(ffn_events, disable_pdl, grid_ctas):
-    opts = DecodeOpts(None, None, int(bool(disable_pdl)), int(grid_ctas))
+def _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns=0, test_starve_first_down=False):
+    opts = DecodeOpts(None, None, int(bool(disable_pdl)), int(grid_ctas), int(wait_limit_ns),
+                      int(bool(test_starve_first_down)), 0)
     if ffn_events is not None:
         opts.ffn_begin = ctypes.c_void_p(ffn_events[0].cuda_event)
         opts.ffn_end = ctypes.c_void_p(ffn_events[1].cuda_event)
@@ -266,16 +269,19 @@ def _opts(ffn_events, disable_pdl, grid_ctas):
 
 def slimwise_moe_decode_ex(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
                            out=None, workspace=None, stream=None, ffn_events=None,
-                           disable_pdl=False, grid_ctas=0):
+                           disable_pdl=False, grid_ctas=0, wait_limit_ns=0,
+                           test_starve_first_down=False):
     """slimwise_moe_decode with launch options; retained_idx None = full pool.
 
     ffn_events: optional (begin, end) torch.cuda.Event pair recorded around the
-    expert-FFN kernel on the launch stream.
+    expert-FFN kernel on the launch stream.  wait_limit_ns: limit of the FFN
+    kernel's bounded waits (0: 1 s).  test_starve_first_down: tests only, makes
+    the first down item's dependency wait run out.
     """
     s, out, workspace = _prep(hidden, router_w, w_gate_up, w_down, top_k, out, workspace)
     if retained_idx is not None:
         _dev(retained_idx, torch.int32, "retained_idx")
-    opts = _opts(ffn_events, disable_pdl, grid_ctas)
+    opts = _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns, test_starve_first_down)
     n_ret = 0 if retained_idx is None else int(retained_idx.numel())
     _check(load().slimwise_moe_decode_ex(
         _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),

@@ -229,9 +229,13 @@ struct FfnMaps {
   CUtensorMap act_s[kTokBoxSizes];  // [B rows, Is cols] bf16, token order
 };
 
+// timeout_ns: limit of every bounded wait; starve_first_down (tests only):
+// the first routed down item waits for a gate/up tile that never exists.
+constexpr uint64_t kDefaultWaitLimitNs = 1000000000ull;
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
                               __nv_bfloat16 *out, int grid, bool pdl,
-                              cudaStream_t stream);
+                              cudaStream_t stream, uint64_t timeout_ns = kDefaultWaitLimitNs,
+                              int starve_first_down = 0);
 
 // Importance statistics of the last full-pool call in `ws` added to stats
 // (fp64 [E, 4]); retained set from statistics (criterion 0 mass, 1 EAN, 2 REAP).

@@ -33,9 +33,12 @@
 //            At 32 or more tokens per retained expert it combines 8 of its
 //            tokens itself and queues the rest in the workspace; epilogue
 //            groups with no items left drain that queue.
-// Every wait is bounded (1 s): on timeout the CTA records an error bit in the
-// workspace, stops taking work, drains its own copies and MMAs, frees TMEM
-// and exits.
+// Every wait is bounded (1 s unless the caller sets another limit): on
+// timeout the CTA records an error bit in the workspace, stops taking work,
+// drains its own copies and MMAs, frees TMEM and exits.  The 128 threads of an
+// epilogue group take each wait's outcome together (a barrier reduction), so
+// a wait that completes just as another thread gives up cannot split the
+// group between its named barrier and the exit.
 #include "common.cuh"
 
 namespace slimwise {
@@ -52,7 +55,6 @@ constexpr int kGroupMiscInts = 2 + kMaxTokTile;
 // tokens a down item's epilogue combines itself; the rest of its list goes
 // to the grid-wide combine queue
 constexpr int kInlineCombines = 2 * kEpiThreads / 32;
-constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 // 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
 #ifndef SLIMWISE_STAGE_SUB
@@ -209,6 +211,20 @@ __device__ __forceinline__ void epi_bar(int g) {
   asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kEpiThreads) : "memory");
 }
 
+// The same barrier, returning whether `v` holds on every thread of group g.
+__device__ __forceinline__ bool epi_all(int g, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.and.pred p, %2, %3, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "r"(1 + g), "n"(kEpiThreads)
+      : "memory");
+  return r != 0;
+}
+
 __device__ __forceinline__ int ld_acquire(const int *p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -227,7 +243,8 @@ template <bool kShared>
 __global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
-                      int tmem_cols, int static_first) {
+                      int tmem_cols, int static_first, uint64_t timeout_ns,
+                      int starve_first_down) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -359,7 +376,7 @@ __global__ void __maxnreg__(128)
                                atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
         first = false;
         if (*abort) item = 0x7FFFFFFF;
-        if (!mbar_wait_bounded(ite_bar(slot), rphase ^ 1u, abort, kTimeoutNs)) {
+        if (!mbar_wait_bounded(ite_bar(slot), rphase ^ 1u, abort, timeout_ns)) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
           break;
         }
@@ -379,13 +396,16 @@ __global__ void __maxnreg__(128)
         if (it.down) {
           // the entry's activations must be complete: all its gate/up tiles
           const int *done = &ws.entry_done[it.entry];
-          const int need = (kShared && it.shared) ? ip.t1s : t1;
+          int need = (kShared && it.shared) ? ip.t1s : t1;
+          // test only: the first routed down item waits for one gate/up tile
+          // more than exist, so its wait runs out (the timeout path)
+          if (starve_first_down && item == ip.S * ip.t1s + ip.r1) ++need;
           bool ok = ld_acquire(done) >= need;
           if (!ok) {
             const uint64_t t0 = global_timer_ns();
             while (!(ok = ld_acquire(done) >= need)) {
               if (*abort) break;
-              if (global_timer_ns() - t0 > kTimeoutNs) {
+              if (global_timer_ns() - t0 > timeout_ns) {
                 raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
                 break;
               }
@@ -424,7 +444,7 @@ __global__ void __maxnreg__(128)
         const uint32_t sub_bytes = (uint32_t)(kATileBytes + (kTokBox << box_m) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
-          if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, kTimeoutNs)) {
+          if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, timeout_ns)) {
             if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
             ok = false;
             break;
@@ -466,7 +486,7 @@ __global__ void __maxnreg__(128)
       int n_consumed = 0;
       bool issued_any = false;
       for (int local = 0;; ++local) {
-        if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, kTimeoutNs)) {
+        if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, timeout_ns)) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
           break;
         }
@@ -480,7 +500,7 @@ __global__ void __maxnreg__(128)
         const Item it = decode_item<kShared>(item, ip, ws);
         const int b = local & 1;
         const uint32_t use = (uint32_t)(local >> 1);
-        if (!mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, kTimeoutNs)) {
+        if (!mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, timeout_ns)) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
           break;
         }
@@ -492,7 +512,7 @@ __global__ void __maxnreg__(128)
         const int nk = (nsub_total + kStageSub - 1) / kStageSub;
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
-          if (!mbar_wait_bounded(full_bar(stage), phase, abort, kTimeoutNs)) {
+          if (!mbar_wait_bounded(full_bar(stage), phase, abort, timeout_ns)) {
             if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
             ok = false;
             break;
@@ -548,10 +568,9 @@ __global__ void __maxnreg__(128)
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
-      if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, kTimeoutNs)) {
-        if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
-        break;
-      }
+      bool got = mbar_wait_bounded(itf_bar(slot), rphase, abort, timeout_ns);
+      if (!got && !*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+      if (!epi_all(g, got)) break;
       const int item = ring[slot];
       mbar_arrive(ite_bar(slot));
       if (++slot == kItemRing) {
@@ -563,10 +582,9 @@ __global__ void __maxnreg__(128)
       if (b != g) continue;
       const Item it = decode_item<kShared>(item, ip, ws);
       const uint32_t use = (uint32_t)(local >> 1);
-      if (!mbar_wait_bounded(accf_bar(b), use & 1u, abort, kTimeoutNs)) {
-        if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
-        break;
-      }
+      got = mbar_wait_bounded(accf_bar(b), use & 1u, abort, timeout_ns);
+      if (!got && !*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+      if (!epi_all(g, got)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * nb_cols);
       if (!it.down) {
@@ -685,7 +703,7 @@ __global__ void __maxnreg__(128)
   // Every warp with no work left (producer, MMA issuer and the epilogue
   // groups) takes queued combines, one slot at a time, until it draws a
   // closed slot.
-  while (comb_queue && !*abort && total_down > 0) {
+  while (comb_queue && total_down > 0 && !__any_sync(0xFFFFFFFFu, *abort != 0)) {
     int v = -1;
     if (lane == 0) {
       const int h = atomicAdd(&ws.ctrl[kCtrlCombHead], 1);
@@ -699,7 +717,7 @@ __global__ void __maxnreg__(128)
             break;
           }
           if (*abort) break;
-          if (global_timer_ns() - t0 > kTimeoutNs) {
+          if (global_timer_ns() - t0 > timeout_ns) {
             raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
             break;
           }
@@ -740,7 +758,8 @@ int ffn_stages_for(int tok_chunk, size_t smem_limit) {
 
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
                               __nv_bfloat16 *out, int grid, bool pdl,
-                              cudaStream_t stream) {
+                              cudaStream_t stream, uint64_t timeout_ns,
+                              int starve_first_down) {
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
@@ -780,7 +799,8 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   // items are assigned statically to first CTAs only if all of them are
   // resident at once (a down item may wait on another CTA's first item)
   const int static_first = grid <= sms ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols, static_first);
+  return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols, static_first,
+                            timeout_ns, starve_first_down);
 }
 
 }  // namespace slimwise

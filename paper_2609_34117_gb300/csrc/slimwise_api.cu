@@ -250,8 +250,12 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
   const bool timed = opts && opts->ffn_begin && opts->ffn_end;
   if (timed && cudaEventRecord(static_cast<cudaEvent_t>(opts->ffn_begin), st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
+  const uint64_t wait_limit = (opts && opts->wait_limit_ns > 0)
+                                  ? (uint64_t)opts->wait_limit_ns
+                                  : kDefaultWaitLimitNs;
+  const int starve = (opts && opts->test_starve_first_down) ? 1 : 0;
   if (launch_expert_ffn(maps, d, w, static_cast<__nv_bfloat16 *>(out), grid,
-                        pdl && !timed, st) != cudaSuccess)
+                        pdl && !timed, st, wait_limit, starve) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   if (timed && cudaEventRecord(static_cast<cudaEvent_t>(opts->ffn_end), st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;

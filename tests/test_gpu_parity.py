@@ -209,7 +209,7 @@ def test_compact_checkpoint_equals_masked_pool(qwen, m_prime):
     _check_out(compact.float().cpu().numpy()[tokens], ref["out"])
     # and mapped back to original ids it is the masked pool's routing
     ref_m = oracle.route(oracle.router_logits(xb, qwen.wr.numpy()), retained.cpu().numpy(), 8)
-    assert np.array_equal(ids.numpy()[ref["idx"]], ref_m[0])
+    assert np.array_equal(ids.cpu().numpy()[ref["idx"]], ref_m[0])
 
 
 class SharedExpert:
