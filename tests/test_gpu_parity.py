@@ -281,6 +281,25 @@ def test_shared_expert_closed_gate_is_the_routed_layer(tiny, tiny_shared):
     assert torch.equal(with_se, routed)
 
 
+@pytest.mark.parametrize("B,m_prime,hot", [(128, None, 1), (200, None, 2), (256, 8, 1)])
+def test_hot_expert_spans_several_slots(B, m_prime, hot):
+    # One or two experts chosen by every token, the rest of the load spread
+    # thin: the token chunk follows the mean load (16 or 128 rows), so a hot
+    # expert becomes several work entries, each streaming the expert's weight
+    # tiles for its own chunk of tokens.  (256, 8): the combine queue is in
+    # use too.
+    shape = synth.LayerShape(hidden=256, num_experts=64, inter=128, top_k=2)
+    layer = Layer(shape, seed=11)
+    retained = None if m_prime is None else synth.retained_set(64, m_prime, 13)
+    hot_ids = [5, 17] if retained is None else [int(retained[2])]
+    bias = torch.zeros(64)
+    for j, e in enumerate(hot_ids[:hot]):
+        bias[e] = 8.0 - 2.0 * j
+    x, wr = synth.apply_popularity_bias(synth.hidden_states(B, shape, 140 + B), layer.wr, bias)
+    _, _, route = _case(layer, B=B, m_prime=m_prime, seed_x=140 + B, seed_imp=13, x=x, wr=wr)
+    assert route["counts"].max() == B
+
+
 @pytest.mark.parametrize("B", [1, 5, 17, 33, 300])
 def test_ragged_batches_and_token_chunks(tiny, B):
     # k = m' = 8: every token selects every retained expert, so each expert
