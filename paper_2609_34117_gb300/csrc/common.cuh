@@ -6,6 +6,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <math.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -21,40 +22,39 @@ constexpr int kTileRows = 128;       // MMA M: weight rows per work item
 constexpr int kGateRows = 64;        // gate rows (and as many up rows) per gate/up item
 constexpr int kMaxTokTile = 256;     // MMA N limit: tokens of one expert per item
 constexpr int kTokBox = 16;          // token rows per MMA N step
-constexpr int kTokBoxSizes = 5;      // token-row TMA boxes of kTokBox << m rows, m < 5
+constexpr int kTokBoxSizes = 16;     // token-row TMA boxes of kTokBox * (m + 1) rows, m < 16
 constexpr int kATileBytes = kTileRows * kBlockK * 2;   // 16 KiB
 constexpr int kMaxExperts = 1024;
 constexpr int kMaxTopK = 32;
 constexpr int kCombineTile = 128;    // h values per down item (= kTileRows)
 
 // Tokens of one expert handled by one work item (the FFN kernel's largest
-// MMA N): a power of two from 16 to 256, so that one TMA box of a power-of-two
-// height carries an item's token rows.  It is sized to twice the mean load of
-// a retained expert (B*k/m' selections) rather than to the largest possible
-// load (B): each pipeline stage holds a chunk of token rows, so a smaller
-// chunk leaves room for more weight tiles in flight.  An expert with more
-// tokens than a chunk becomes several entries; their items are handed out
-// together, so the repeated weight reads come from L2.
+// MMA N): a multiple of 16 from 16 to 256; one TMA box of 16 n rows carries
+// an item's n16 = n groups of token rows.  Each pipeline stage holds a chunk
+// of token rows, so a smaller chunk leaves room for more weight tiles in
+// flight.  The chunk covers the mean load of a retained expert (B*k/m'
+// selections) plus three standard deviations of a binomial load, and never
+// more than twice the mean, rather than the largest possible load (B).  An
+// expert with more tokens than a chunk becomes several entries; their items
+// are handed out together, so the repeated weight reads come from L2.
 __host__ __device__ inline int pow2_at_least(int v) {
   int p = 1;
   while (p < v) p <<= 1;
   return p;
 }
+__host__ __device__ inline int round16(int v) { return (v + kTokBox - 1) / kTokBox * kTokBox; }
 __host__ __device__ inline int token_chunk_for(int B, int k, int m_ret) {
-  int most = pow2_at_least(B);  // an expert is selected at most once per token
+  int most = round16(B);  // an expert is selected at most once per token
   if (most < kTokBox) most = kTokBox;
   if (most > kMaxTokTile) most = kMaxTokTile;
-  const int mean = (B * k + m_ret - 1) / m_ret;
-  int c = pow2_at_least(2 * mean);
+  const float mean = (float)B * (float)k / (float)m_ret;
+  const float spread = mean + 3.0f * sqrtf(mean);
+  int c = round16((int)ceilf(spread < 2.0f * mean ? spread : 2.0f * mean));
   if (c < kTokBox) c = kTokBox;
   return c < most ? c : most;
 }
-// Index m of the token box (kTokBox << m rows) that covers n16 16-row groups.
-__host__ __device__ inline int token_box_for(int n16) {
-  int m = 0;
-  while ((1 << m) < n16) ++m;
-  return m;
-}
+// Index m of the token box (kTokBox * (m + 1) rows) that covers n16 16-row groups.
+__host__ __device__ inline int token_box_for(int n16) { return n16 - 1; }
 constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
 // Tokens per routing cluster.  Up to 4 a routing CTA stages its hidden rows
 // in under 17 KiB of shared memory and fits beside a persistent expert-FFN
@@ -204,7 +204,7 @@ inline Ws make_ws(void *base, const WsLayout &L) {
 struct Dims {
   int B, H, E, I, k;
   int m_ret;      // retained experts (E for the full pool)
-  int tok_chunk;  // max tokens of one expert per work item (power of two, 16..256)
+  int tok_chunk;  // max tokens of one expert per work item (multiple of 16, 16..256)
   int Is;         // shared-expert intermediate width (0: no shared expert)
   int S;          // shared-expert work entries: ceil(B / tok_chunk), 0 without one
 };
@@ -220,8 +220,8 @@ cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shar
 struct FfnMaps {
   CUtensorMap w_gu;                 // [E*2I rows, H cols] bf16, box 64 x 64
   CUtensorMap w_down;               // [E*H rows, I cols] bf16, box 64 x 64
-  CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16, box 64 x (16 << m)
-  CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16, box 64 x (16 << m)
+  CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16, box 64 x 16 (m + 1)
+  CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16, box 64 x 16 (m + 1)
   // shared expert (encoded only when there is one)
   CUtensorMap w_gu_s;               // [2Is rows, H cols] bf16, box 64 x 64
   CUtensorMap w_down_s;             // [H rows, Is cols] bf16, box 64 x 64

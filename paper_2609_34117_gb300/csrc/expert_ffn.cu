@@ -289,7 +289,7 @@ __global__ void __maxnreg__(128)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&maps.w_gu);
     tma_prefetch_desc(&maps.w_down);
-    for (int m = 0; m < kTokBoxSizes && (kTokBox << m) <= d.tok_chunk; ++m) {
+    for (int m = 0; m < kTokBoxSizes && kTokBox * (m + 1) <= d.tok_chunk; ++m) {
       tma_prefetch_desc(&maps.xp[m]);
       tma_prefetch_desc(&maps.act[m]);
       if constexpr (kShared) {
@@ -415,8 +415,8 @@ __global__ void __maxnreg__(128)
           if (!ok) break;
           fence_proxy_async_global();
         }
-        // the item's token rows: one box of the power-of-two height that
-        // covers them (rows past the entry are loaded but not multiplied)
+        // the item's token rows: one box of the tokens rounded up to 16
+        // rows (rows past the entry are loaded but not multiplied)
         const int box_m = token_box_for(it.n16);
         int nsub_total, row0, row1;
         const void *amap;
@@ -441,7 +441,7 @@ __global__ void __maxnreg__(128)
           }
         }
         const int nk = (nsub_total + kStageSub - 1) / kStageSub;
-        const uint32_t sub_bytes = (uint32_t)(kATileBytes + (kTokBox << box_m) * kBlockK * 2);
+        const uint32_t sub_bytes = (uint32_t)(kATileBytes + kTokBox * (box_m + 1) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, timeout_ns)) {
@@ -768,10 +768,10 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   if (err != cudaSuccess) return err;
   err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (err != cudaSuccess) return err;
-  // the token maps exist for boxes of 16 << m <= tok_chunk rows, and an
-  // entry's box covers at most tok_chunk rows: tok_chunk must be a power of
-  // two in [16, 256]
-  if (d.tok_chunk < kTokBox || d.tok_chunk > kMaxTokTile || (d.tok_chunk & (d.tok_chunk - 1)))
+  // the token maps exist for boxes of 16 (m + 1) <= tok_chunk rows, and an
+  // entry's box covers at most tok_chunk rows: tok_chunk must be a multiple
+  // of 16 in [16, 256]
+  if (d.tok_chunk < kTokBox || d.tok_chunk > kMaxTokTile || d.tok_chunk % kTokBox != 0)
     return cudaErrorInvalidValue;
   // leave room on each SM for the next layer's routing CTAs, which become
   // resident while this grid finishes (programmatic dependent launch), where

@@ -149,56 +149,67 @@ struct SharedExpert {
   int32_t inter;          // Is
 };
 
-struct MapsKey {
-  const void *w_gu, *w_down, *xp, *act, *gu_s, *down_s;
-  int E, H, I, Is, B, tok_chunk;
+// The weight maps depend on the weight tensors only; the token maps on the
+// workspace, the batch and the token chunk.  They are cached separately, so
+// that rotating between weight copies re-encodes two or four maps, not the
+// token maps of every box height.
+struct WeightMapsKey {
+  const void *w_gu, *w_down, *gu_s, *down_s;
+  int E, H, I, Is, device;
+  bool operator==(const WeightMapsKey &o) const {
+    return w_gu == o.w_gu && w_down == o.w_down && gu_s == o.gu_s && down_s == o.down_s &&
+           E == o.E && H == o.H && I == o.I && Is == o.Is && device == o.device;
+  }
+};
+struct TokenMapsKey {
+  const void *xp, *act, *xt, *act_s;
+  int H, I, Is, B, tok_chunk, device;
   uint64_t slots;
-  int device;
-  bool operator==(const MapsKey &o) const {
-    return w_gu == o.w_gu && w_down == o.w_down && xp == o.xp && act == o.act &&
-           gu_s == o.gu_s && down_s == o.down_s && E == o.E && H == o.H && I == o.I &&
-           Is == o.Is && B == o.B && tok_chunk == o.tok_chunk && slots == o.slots &&
-           device == o.device;
+  bool operator==(const TokenMapsKey &o) const {
+    return xp == o.xp && act == o.act && xt == o.xt && act_s == o.act_s && H == o.H &&
+           I == o.I && Is == o.Is && B == o.B && tok_chunk == o.tok_chunk &&
+           device == o.device && slots == o.slots;
   }
 };
 
 bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, const Ws &w,
                   const Dims &d, uint64_t slots, const SharedExpert &se) {
-  thread_local bool have = false;
-  thread_local MapsKey last;
-  thread_local FfnMaps cached;
+  thread_local bool have_w = false, have_t = false;
+  thread_local WeightMapsKey last_w;
+  thread_local TokenMapsKey last_t;
+  thread_local FfnMaps cached;  // both halves of the last call on this thread
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  const MapsKey key = {w_gate_up, w_down, w.xp, w.act, se.gate_up, se.down,
-                       d.E, d.H, d.I, d.Is, d.B, d.tok_chunk, slots, dev};
-  if (have && key == last) {
-    *maps = cached;
-    return true;
+  const WeightMapsKey kw = {w_gate_up, w_down, se.gate_up, se.down, d.E, d.H, d.I, d.Is, dev};
+  const TokenMapsKey kt = {w.xp, w.act, w.xt, w.act_s, d.H, d.I, d.Is, d.B, d.tok_chunk, dev, slots};
+  if (!(have_w && kw == last_w)) {
+    have_w = false;
+    if (encode_map(&cached.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
+        encode_map(&cached.w_down, w_down, (uint64_t)d.E * d.H, d.I, kGateRows))
+      return false;
+    if (d.Is > 0 &&
+        (encode_map(&cached.w_gu_s, se.gate_up, 2 * (uint64_t)d.Is, d.H, kGateRows) ||
+         encode_map(&cached.w_down_s, se.down, (uint64_t)d.H, d.Is, kGateRows)))
+      return false;
+    last_w = kw;
+    have_w = true;
   }
-  have = false;
-  FfnMaps m;
-  std::memset(&m, 0, sizeof(m));
-  if (encode_map(&m.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
-      encode_map(&m.w_down, w_down, (uint64_t)d.E * d.H, d.I, kGateRows))
-    return false;
-  // token boxes up to the chunk: an item's box covers at most chunk rows
-  for (int b = 0; b < kTokBoxSizes && (kTokBox << b) <= d.tok_chunk; ++b)
-    if (encode_map(&m.xp[b], w.xp, slots, d.H, kTokBox << b) ||
-        encode_map(&m.act[b], w.act, slots, d.I, kTokBox << b))
-      return false;
-  if (d.Is > 0) {
-    if (encode_map(&m.w_gu_s, se.gate_up, 2 * (uint64_t)d.Is, d.H, kGateRows) ||
-        encode_map(&m.w_down_s, se.down, (uint64_t)d.H, d.Is, kGateRows))
-      return false;
-    for (int b = 0; b < kTokBoxSizes && (kTokBox << b) <= d.tok_chunk; ++b)
-      if (encode_map(&m.xt[b], w.xt, (uint64_t)d.B, d.H, kTokBox << b) ||
-          encode_map(&m.act_s[b], w.act_s, (uint64_t)d.B, d.Is, kTokBox << b))
+  if (!(have_t && kt == last_t)) {
+    have_t = false;
+    // token boxes up to the chunk: an item's box covers at most chunk rows
+    for (int b = 0; b < kTokBoxSizes && kTokBox * (b + 1) <= d.tok_chunk; ++b) {
+      const uint32_t rows = (uint32_t)(kTokBox * (b + 1));
+      if (encode_map(&cached.xp[b], w.xp, slots, d.H, rows) ||
+          encode_map(&cached.act[b], w.act, slots, d.I, rows))
         return false;
+      if (d.Is > 0 && (encode_map(&cached.xt[b], w.xt, (uint64_t)d.B, d.H, rows) ||
+                       encode_map(&cached.act_s[b], w.act_s, (uint64_t)d.B, d.Is, rows)))
+        return false;
+    }
+    last_t = kt;
+    have_t = true;
   }
-  cached = m;
-  last = key;
-  have = true;
-  *maps = m;
+  *maps = cached;
   return true;
 }
 
