@@ -56,18 +56,14 @@ __host__ __device__ inline int token_chunk_for(int B, int k, int m_ret) {
 // Index m of the token box (kTokBox * (m + 1) rows) that covers n16 16-row groups.
 __host__ __device__ inline int token_box_for(int n16) { return n16 - 1; }
 constexpr int kMinTokChunk = 16;     // smallest token_chunk_for(): bounds the entry count
-// Tokens per routing cluster.  Up to 4 a routing CTA stages its hidden rows
-// in under 17 KiB of shared memory and fits beside a persistent expert-FFN
-// CTA; with 8 or 16 it stages 64 KiB and never does.  One wave of routing
-// CTAs (two per SM) holds 38 clusters: above 152 tokens clusters of 4 need
-// two waves, so pools of at most 64 retained experts (small slices per CTA)
-// take 8 tokens per cluster there; above 304 tokens every pool takes 16,
-// staged as bf16.
+// Tokens per routing cluster.  One wave of routing CTAs (two per SM) holds
+// 38 clusters: above 152 tokens clusters of 4 need two waves, so every pool
+// takes 8 tokens per cluster there; above 304 tokens 16, staged as bf16.
 inline int route_tokens_per_cluster(int B, int m_ret) {
+  (void)m_ret;
   if (B <= 32) return 1;
   if (B <= 64) return 2;
   if (B <= 152) return 4;
-  if (B <= 256) return m_ret <= 64 ? 8 : 4;
   return B <= 304 ? 8 : 16;
 }
 
@@ -80,9 +76,6 @@ enum CtrlWord {
   kCtrlWorkCounter = 4, // dynamic scheduler counter
   kCtrlErr = 5,         // SLIMWISE_DEVERR_* bits of the current call
   kCtrlTraceStep = 6,   // step counter of the optional trace ring
-  kCtrlCombTail = 7,    // (token, h tile) combines queued by the FFN kernel
-  kCtrlCombHead = 8,    // queue slots taken by combining warps
-  kCtrlDownDone = 9,    // down items whose epilogue has finished
   kCtrlWords = 16
 };
 
@@ -98,7 +91,7 @@ enum TraceSlot {
 // Byte offsets of every workspace region (all 1024-byte aligned).
 struct WsLayout {
   size_t ctrl, topk_idx, topk_gate, counts, offsets, union_ids, entries,
-      entry_done, perm, pos, comb_cnt, comb_q, xp, act, y, shared_gate, xt, act_s, y_s, total;
+      entry_done, perm, pos, xp, act, y, shared_gate, xt, act_s, y_s, total;
   int32_t max_entries;
 };
 
@@ -136,8 +129,6 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
   L.entry_done = take((size_t)L.max_entries * 4);
   L.perm = take(slots * 4);
   L.pos = take(slots * 4);
-  L.comb_cnt = take((size_t)B * (H / kCombineTile) * 4);
-  L.comb_q = take((size_t)B * (H / kCombineTile) * 4);
   L.xp = take(slots * H * 2);
   L.act = take(slots * I * 2);
   L.y = take(slots * H * 4);
@@ -165,8 +156,6 @@ struct Ws {
   int32_t *entry_done; // gate/up items finished per entry
   int32_t *perm;
   int32_t *pos;
-  int32_t *comb_cnt;   // [B, H/128] down items finished per (token, h tile)
-  int32_t *comb_q;     // [B * H/128] queued combines, 1 + t * (H/128) + tile; 0 = empty
   __nv_bfloat16 *xp;   // [B*k, H] hidden rows in grouped order
   __nv_bfloat16 *act;  // [B*k, I] SwiGLU activations in grouped order
   float *y;            // [B*k, H] expert outputs in grouped order
@@ -189,8 +178,6 @@ inline Ws make_ws(void *base, const WsLayout &L) {
   w.entry_done = (int32_t *)(b + L.entry_done);
   w.perm = (int32_t *)(b + L.perm);
   w.pos = (int32_t *)(b + L.pos);
-  w.comb_cnt = (int32_t *)(b + L.comb_cnt);
-  w.comb_q = (int32_t *)(b + L.comb_q);
   w.xp = (__nv_bfloat16 *)(b + L.xp);
   w.act = (__nv_bfloat16 *)(b + L.act);
   w.y = (float *)(b + L.y);
@@ -232,6 +219,9 @@ struct FfnMaps {
 // timeout_ns: limit of every bounded wait; starve_first_down (tests only):
 // the first routed down item waits for a gate/up tile that never exists.
 constexpr uint64_t kDefaultWaitLimitNs = 1000000000ull;
+// The gate-weighted combine of every (token, 128-column tile), after the
+// expert FFN.
+cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStream_t stream);
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
                               __nv_bfloat16 *out, int grid, bool pdl,
                               cudaStream_t stream, uint64_t timeout_ns = kDefaultWaitLimitNs,

@@ -1,5 +1,5 @@
 // expert_ffn.cu -- grouped SwiGLU expert FFN over the selected-expert union,
-// with the gate-weighted combine fused into its epilogue.
+// and the gate-weighted combine of its outputs (a second, small kernel).
 //
 // Decode reads the weights of every expert in the union of the batch's
 // selections once per step (SlimWise Sec. 2.1, Eq. 1) and each expert sees
@@ -14,7 +14,7 @@
 //            waits for a down item's activations, and issues each stage's
 //            copies -- the 128-row weight tile (two 64-row boxes) and the
 //            item's token rows (one box, its height the token count rounded
-//            up to a power of two).  The issuing thread's copy rate bounds
+//            up to 16 rows).  The issuing thread's copy rate bounds
 //            the stage rate, so a stage takes three copies whatever the
 //            number of tokens, and the descriptors are chosen once per item.
 //   warp 1   MMA issuer (one thread) and TMEM owner; double-buffered
@@ -28,11 +28,13 @@
 //            stores bf16 act in grouped order and counts the tile done.
 //   down    (entry, h-tile): A = 128 rows of W_down[e], K = I, B = act of the
 //            entry's tokens (after all its gate/up tiles are done); epilogue
-//            stores fp32 y; the last of the k contributions to a
-//            (token, h-tile) sums sum_j g[t,j] y_j in j order and writes bf16.
-//            At 32 or more tokens per retained expert it combines 8 of its
-//            tokens itself and queues the rest in the workspace; epilogue
-//            groups with no items left drain that queue.
+//            stores fp32 y in grouped order.
+// The combine kernel runs next on the stream (programmatic dependent launch:
+// its CTAs become resident beside this grid's last CTAs): one warp per
+// (token, 128-column tile) sums g[t,j] y_j in j order and writes bf16.  With
+// the whole GPU's warps on it the combine takes a few microseconds after the
+// last expert output, where combining inside this kernel left it to the few
+// CTAs that finished the last items.
 // Every wait is bounded (1 s unless the caller sets another limit): on
 // timeout the CTA records an error bit in the workspace, stops taking work,
 // drains its own copies and MMAs, frees TMEM and exits.  The 128 threads of an
@@ -49,12 +51,6 @@ constexpr int kFfnThreads = 64 + kEpiGroups * kEpiThreads;
 constexpr int kItemRing = 4;
 constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
 constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
-constexpr int kEpiWarps = kEpiThreads / 32;
-// per epilogue group: combine count, queue base and token list
-constexpr int kGroupMiscInts = 2 + kMaxTokTile;
-// tokens a down item's epilogue combines itself; the rest of its list goes
-// to the grid-wide combine queue
-constexpr int kInlineCombines = 2 * kEpiThreads / 32;
 
 // 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
 #ifndef SLIMWISE_STAGE_SUB
@@ -78,8 +74,8 @@ __host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
   p.bar_off = p.xch_off + kXchBytes;
   // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
   p.misc_off = p.bar_off + 8 * (2 * stages + 4 + 2 * kItemRing + 1);
-  // item ring, tmem base, abort, consumed stages, then per epilogue group
-  p.total = p.misc_off + 4 * (kItemRing + 3) + 4 * kEpiGroups * kGroupMiscInts + 1024;
+  // item ring, tmem base, abort, consumed stages
+  p.total = p.misc_off + 4 * (kItemRing + 3) + 1024;
   return p;
 }
 
@@ -198,14 +194,6 @@ __device__ __forceinline__ void combine_token(const Ws &ws, const Dims &d,
                  *reinterpret_cast<const uint32_t *>(&hi));
 }
 
-// The combine queue pays where the combine lists are long, at 32 or more
-// tokens per retained expert on average; below that its end-of-launch
-// handshake (the last down item closes the queue, the waiting warps see it)
-// costs more than the combines it spreads.
-__device__ __forceinline__ bool use_combine_queue(const Dims &d) {
-  return d.B * d.k >= 32 * d.m_ret;
-}
-
 // Named barrier of epilogue group g (ids 1.., id 0 is __syncthreads).
 __device__ __forceinline__ void epi_bar(int g) {
   asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kEpiThreads) : "memory");
@@ -237,13 +225,14 @@ __device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit
 }
 
 // At most 128 registers a thread (320 threads: 40 K of the SM's 64 K), so
-// that a routing CTA of the next layer (256 threads, at most 96 registers)
+// that a CTA of the dependent combine kernel (256 threads, 72 registers)
 // can become resident beside this one.
 template <bool kShared>
 __global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
-                      int tmem_cols, int static_first, uint64_t timeout_ns,
+                      int tmem_cols, int static_first, int early_dependents,
+                      uint64_t timeout_ns,
                       int starve_first_down) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
@@ -264,7 +253,6 @@ __global__ void __maxnreg__(128)
   volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc + kItemRing);
   volatile int *abort = misc + kItemRing + 1;
   volatile int *consumed = misc + kItemRing + 2;     // stages the MMA finished with
-  int *group_misc = misc + kItemRing + 3;            // [kEpiGroups][kGroupMiscInts]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -336,6 +324,11 @@ __global__ void __maxnreg__(128)
 
   // Everything below reads the grouping kernel's results.
   pdl_wait_primary();
+  // Above 64 tokens the combine kernel that follows may become resident now
+  // (it waits for this grid to finish): measured 2-4 us faster per step at
+  // B = 128-512, 0.5 us slower at B = 64, where the trigger stays at the end
+  // of the work.
+  if (early_dependents) pdl_launch_dependents();
 #ifdef SLIMWISE_TRACE
   const int tr_step = ws.ctrl[kCtrlTraceStep] - 1;
   if (blockIdx.x == 0 && threadIdx.x == 0) trace_stamp(ws, tr_step, kTrFfnStart);
@@ -352,9 +345,6 @@ __global__ void __maxnreg__(128)
   ip.S = kShared ? d.S : 0;
   const int nb_cols = d.tok_chunk;  // TMEM columns per accumulator buffer
 
-  const int total_down = total - ip.r1 - ip.S * ip.t1s;  // down items of the launch
-  const int q_cap = d.B * t2;                            // combine-queue slots
-  const bool comb_queue = use_combine_queue(d);
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -560,11 +550,6 @@ __global__ void __maxnreg__(128)
     const int row = 32 * q + lane;      // accumulator row = TMEM lane
     const int et = (threadIdx.x - 64) & (kEpiThreads - 1);
     float *xb = xch + g * kTileRows * kXchStride;
-    int *gm = group_misc + g * kGroupMiscInts;
-    int *comb_n = gm;
-    int *q_base = gm + 1;
-    int *comb_list = gm + 2;                          // [kMaxTokTile]
-    const int ew = q;                                 // warp within the group
     int slot = 0;
     uint32_t rphase = 0;
     for (int local = 0;; ++local) {
@@ -644,91 +629,12 @@ __global__ void __maxnreg__(128)
               ybase[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
           }
         }
+        // the expert outputs are all a down item writes: the combine kernel
+        // that follows this grid sums them
         tc_fence_before();
         mbar_arrive(acce_bar(b));
-        __threadfence();
-        if (et == 0) *comb_n = 0;
-        epi_bar(g);
-        // count this contribution for each token; the last of its k routed
-        // (and, with a shared expert, one shared) contributions combines
-        const int last = kShared ? d.k : d.k - 1;
-        for (int col = et; col < it.n; col += kEpiThreads) {
-          const int t = (kShared && it.shared) ? it.slot_base + col
-                                               : __ldcg(&ws.perm[it.slot_base + col]) / d.k;
-          const int old = atomicAdd(&ws.comb_cnt[(size_t)t * t2 + it.tile], 1);
-          if (old == last) comb_list[atomicAdd(comb_n, 1)] = t;
-        }
-        __threadfence();
-        epi_bar(g);
-        const int n_list = *comb_n;
-        // With the combine queue, the first kInlineCombines tokens of the
-        // list are combined here and the rest go to the grid-wide queue,
-        // which every epilogue group drains once it has no items left: the
-        // last experts' items complete most tokens, and their lists would
-        // otherwise be combined one warp round trip at a time on a few CTAs
-        // after all streaming has ended.
-        const int n_inline = comb_queue ? min(n_list, kInlineCombines) : n_list;
-        if (n_list > n_inline) {
-          if (et == 0) *q_base = atomicAdd(&ws.ctrl[kCtrlCombTail], n_list - n_inline);
-          epi_bar(g);
-          const int base = *q_base;
-          // each (token, tile) completes once per call: at most B * t2 slots
-          for (int i = n_inline + et; i < n_list; i += kEpiThreads)
-            if (base + (i - n_inline) < q_cap)
-              ws.comb_q[base + (i - n_inline)] = 1 + comb_list[i] * t2 + it.tile;
-          __threadfence();
-        }
-        for (int i = ew; i < n_inline; i += kEpiWarps)
-          combine_token<kShared>(ws, d, out, comb_list[i], it.tile, lane);
-        // comb_list and comb_n are reused by this group's next down item.
-        // The queued combines are published before the item counts as done;
-        // the launch's last down item then knows the final queue length and
-        // closes every slot past it (-1), which ends the waits below.
-        epi_bar(g);
-        if (comb_queue) {
-          if (et == 0) {
-            __threadfence();
-            const int done = atomicAdd(&ws.ctrl[kCtrlDownDone], 1) + 1;
-            *q_base = done == total_down ? ld_acquire(&ws.ctrl[kCtrlCombTail]) : -1;
-          }
-          epi_bar(g);
-          const int q_final = *q_base;
-          if (q_final >= 0)
-            for (int i = q_final + et; i < q_cap; i += kEpiThreads) ws.comb_q[i] = -1;
-        }
       }
     }
-  }
-
-  // Every warp with no work left (producer, MMA issuer and the epilogue
-  // groups) takes queued combines, one slot at a time, until it draws a
-  // closed slot.
-  while (comb_queue && total_down > 0 && !__any_sync(0xFFFFFFFFu, *abort != 0)) {
-    int v = -1;
-    if (lane == 0) {
-      const int h = atomicAdd(&ws.ctrl[kCtrlCombHead], 1);
-      if (h < q_cap) {
-        const uint64_t t0 = global_timer_ns();
-        uint32_t nap = 64;
-        for (;;) {
-          const int x = ld_acquire(&ws.comb_q[h]);
-          if (x != 0) {
-            v = x;
-            break;
-          }
-          if (*abort) break;
-          if (global_timer_ns() - t0 > timeout_ns) {
-            raise_abort(abort, ws, SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT);
-            break;
-          }
-          __nanosleep(nap);
-          if (nap < 1024) nap <<= 1;
-        }
-      }
-    }
-    v = __shfl_sync(0xFFFFFFFFu, v, 0);
-    if (v <= 0 || v > q_cap) break;
-    combine_token<kShared>(ws, d, out, (v - 1) / t2, (v - 1) % t2, lane);
   }
 
   tc_fence_before();
@@ -747,8 +653,43 @@ __global__ void __maxnreg__(128)
   }
 }
 
-// Shared memory kept free next to one FFN CTA (a routing CTA needs ~10 KiB).
-constexpr size_t kCoResidentSmem = 16 * 1024;
+// The combine of every (token, 128-column tile) after the FFN grid has
+// finished: one warp per pair, the same arithmetic and order as the fused
+// combine (combine_token).  Launched as the FFN's programmatic dependent, so
+// its CTAs become resident beside the FFN's last CTAs and start as soon as
+// the FFN's expert outputs are complete.
+constexpr int kCombineThreads = 256;
+
+template <bool kShared>
+__global__ void __launch_bounds__(kCombineThreads)
+    combine_kernel(Dims d, Ws ws, __nv_bfloat16 *__restrict__ out) {
+  pdl_wait_primary();
+  // the next call's routing may become resident; it waits for this grid
+  pdl_launch_dependents();
+  const int t2 = d.H / kCombineTile;
+  const int lane = threadIdx.x & 31;
+  const int wpc = kCombineThreads / 32;
+  const int pairs = d.B * t2;
+  for (int p = blockIdx.x * wpc + (threadIdx.x >> 5); p < pairs; p += gridDim.x * wpc)
+    combine_token<kShared>(ws, d, out, p / t2, p - (p / t2) * t2, lane);
+}
+
+cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStream_t stream) {
+  const int pairs = d.B * (d.H / kCombineTile);
+  const int wpc = kCombineThreads / 32;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((pairs + wpc - 1) / wpc);
+  cfg.blockDim = dim3(kCombineThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (d.Is > 0) return cudaLaunchKernelEx(&cfg, combine_kernel<true>, d, ws, out);
+  return cudaLaunchKernelEx(&cfg, combine_kernel<false>, d, ws, out);
+}
 
 int ffn_stages_for(int tok_chunk, size_t smem_limit) {
   int s = 12;
@@ -773,11 +714,9 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   // of 16 in [16, 256]
   if (d.tok_chunk < kTokBox || d.tok_chunk > kMaxTokTile || d.tok_chunk % kTokBox != 0)
     return cudaErrorInvalidValue;
-  // leave room on each SM for the next layer's routing CTAs, which become
-  // resident while this grid finishes (programmatic dependent launch), where
-  // they can fit at all: routing CTAs of 8 tokens never do
-  const size_t reserve = route_tokens_per_cluster(d.B, d.m_ret) <= 4 ? kCoResidentSmem : 0;
-  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin - reserve);
+  // the dependent combine kernel needs no shared memory: every byte the
+  // block may opt into goes to pipeline stages
+  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin);
   const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
   auto kernel = d.Is > 0 ? expert_ffn_kernel<true> : expert_ffn_kernel<false>;
@@ -799,8 +738,9 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   // items are assigned statically to first CTAs only if all of them are
   // resident at once (a down item may wait on another CTA's first item)
   const int static_first = grid <= sms ? 1 : 0;
+  const int early_dependents = d.B > 64 ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, stages, tmem_cols, static_first,
-                            timeout_ns, starve_first_down);
+                            early_dependents, timeout_ns, starve_first_down);
 }
 
 }  // namespace slimwise

@@ -191,12 +191,6 @@ __global__ void __launch_bounds__(kGroupThreads)
       }
     }
   }
-  const int ht = H / kCombineTile;
-  for (int i = tid; i < nt * ht; i += blockDim.x) {
-    ws.comb_cnt[(size_t)t0 * ht + i] = 0;
-    ws.comb_q[(size_t)t0 * ht + i] = 0;
-  }
-
   // shared-expert gate of this CTA's tokens: warp w takes token t0 + w; lane
   // l accumulates elements 128c + 4l + q (c, q ascending) with fused
   // multiply-adds, then an xor butterfly over the lanes
@@ -249,9 +243,6 @@ __global__ void __launch_bounds__(kGroupThreads)
     ws.ctrl[kCtrlItems1] = n_entries * t1_items;
     ws.ctrl[kCtrlTotalItems] = n_se * (t1s_items + t2_items) + n_entries * (t1_items + t2_items);
     ws.ctrl[kCtrlWorkCounter] = 0;
-    ws.ctrl[kCtrlCombTail] = 0;
-    ws.ctrl[kCtrlCombHead] = 0;
-    ws.ctrl[kCtrlDownDone] = 0;
   }
   __syncthreads();
   if (blockIdx.x == 0 && tid == 0 && bad) atomicOr(&ws.ctrl[kCtrlErr], bad);

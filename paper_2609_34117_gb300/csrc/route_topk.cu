@@ -87,10 +87,9 @@ __device__ __forceinline__ void fma_chunk2(const XT *xs, int H, int col, float4 
   }
 }
 
-// Hidden rows are staged as fp32 unless that would keep a routing CTA from
-// fitting beside a persistent expert-FFN CTA (about 20 KiB of shared memory
-// are left there): TB = 4 stays bf16; with TB = 8 no routing CTA fits beside
-// one anyway.  TB = 16 stays bf16 too, so that two CTAs fit on an SM.
+// Hidden rows are staged as fp32 (no conversion per use) except at TB = 4
+// and TB = 16, which stage bf16: at 16 tokens so that two CTAs fit on an SM,
+// at 4 because it measured no slower.
 template <int TB>
 struct StageType {
   using T = float;
@@ -126,8 +125,7 @@ __device__ __forceinline__ void take_winner(uint32_t whi, uint32_t wlo, int j, i
 // TB tokens per cluster; NC candidates per lane in the register top-k
 // (m' <= 32 NC), or NC = 0 for the general top-k of larger pools.
 template <int TB, int NC>
-// Two CTAs per SM worth of registers: a routing CTA must fit beside a
-// persistent expert-FFN CTA so it can be resident before that grid ends.
+// Two CTAs per SM worth of registers, so one wave of CTAs holds 38 clusters.
 __global__ void __launch_bounds__(kRouteThreads, 2)
     route_topk_kernel(const __nv_bfloat16 *__restrict__ hidden,
                       const float *__restrict__ router_w,

@@ -1,6 +1,6 @@
 // slimwise_api.cu -- the C ABI declared in include/slimwise_moe.h: argument
-// checks, workspace layout, TMA descriptors, and the three launches of one
-// decode MoE layer (route/top-k -> group/gather -> expert FFN + combine).
+// checks, workspace layout, TMA descriptors, and the four launches of one
+// decode MoE layer (route/top-k -> group/gather -> expert FFN -> combine).
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -267,6 +267,10 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
   const int starve = (opts && opts->test_starve_first_down) ? 1 : 0;
   if (launch_expert_ffn(maps, d, w, static_cast<__nv_bfloat16 *>(out), grid,
                         pdl && !timed, st, wait_limit, starve) != cudaSuccess)
+    return SLIMWISE_ERR_CUDA;
+  // the combine belongs to the timed span: the events bracket the expert FFN
+  // and the combine of its outputs
+  if (launch_combine(d, w, static_cast<__nv_bfloat16 *>(out), pdl, st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   if (timed && cudaEventRecord(static_cast<cudaEvent_t>(opts->ffn_end), st) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;

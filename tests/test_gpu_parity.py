@@ -286,8 +286,8 @@ def test_hot_expert_spans_several_slots(B, m_prime, hot):
     # One or two experts chosen by every token, the rest of the load spread
     # thin: the token chunk follows the mean load (16 or 128 rows), so a hot
     # expert becomes several work entries, each streaming the expert's weight
-    # tiles for its own chunk of tokens.  (256, 8): the combine queue is in
-    # use too.
+    # tiles for its own chunk of tokens.  (256, 8): 64 tokens per retained
+    # expert on average, three entries for the hot one.
     shape = synth.LayerShape(hidden=256, num_experts=64, inter=128, top_k=2)
     layer = Layer(shape, seed=11)
     retained = None if m_prime is None else synth.retained_set(64, m_prime, 13)
@@ -315,8 +315,7 @@ def test_top_k_extremes(tiny, k):
 @pytest.mark.parametrize("B,k", [(33, 12), (300, 16)])
 def test_top_k_above_8(tiny, B, k):
     # the full tiny pool (16 experts) with k > 8: every combine sums two
-    # batches of selections, and at B = 300 (k * B >= 32 m') the combine
-    # queue is in use
+    # batches of selections; at B = 300 most experts hold two work entries
     _case(tiny, B=B, m_prime=None, seed_x=50 + k, seed_imp=0, k=k)
 
 
@@ -329,7 +328,7 @@ def test_top_k_32_qwen(qwen):
 def test_generic_shape(B):
     # H = 640 (five 128-wide chunks: ragged batches of router-row loads, five
     # combine tiles), I = 192 (three gate/up tiles), 24 experts, top-3 of 12;
-    # B = 200 puts the combine queue in use
+    # B = 200 gives token chunks of 80 rows (not a power of two)
     layer = Layer(synth.LayerShape(hidden=640, num_experts=24, inter=192, top_k=3), seed=3)
     _case(layer, B=B, m_prime=12, seed_x=70 + B, seed_imp=4)
 
@@ -418,9 +417,8 @@ def test_workspace_contents_do_not_matter(tiny):
 @pytest.mark.parametrize("fill", [0xFF, 0x00])
 def test_long_combine_lists_all_outputs(tiny, fill):
     # 600 tokens, k = 4 of m' = 8: 300 tokens per retained expert, two work
-    # entries each, so most (token, h tile) combines are completed by items
-    # with long lists and go through the grid-wide combine queue; a workspace
-    # of 0xFF bytes (queue slots reading as closed) must not change anything
+    # entries each, and 2,400 (token, h tile) combines; a workspace of 0xFF
+    # or 0x00 bytes must not change anything
     shape = tiny.shape
     B, k = 600, 4
     x = synth.hidden_states(B, shape, 21)
@@ -436,10 +434,10 @@ def test_long_combine_lists_all_outputs(tiny, fill):
 
 
 @pytest.mark.parametrize("B", [127, 128])
-def test_combine_queue_threshold(tiny, B):
-    # k = 2 of m' = 8: the grid-wide combine queue is used from B * k = 32 m'
-    # (B = 128) on; one token below it every combine is done by the item that
-    # completes it.  Both sides match the oracle on every output.
+def test_combine_grid_ragged_and_full(tiny, B):
+    # k = 2 of m' = 8: B * H/128 (token, tile) combines, one per warp of the
+    # combine kernel's 8-warp CTAs -- a ragged last CTA at B = 127, full CTAs
+    # at B = 128.  Every output against the oracle.
     _case(tiny, B=B, m_prime=8, seed_x=31 + B, seed_imp=6, k=2)
 
 

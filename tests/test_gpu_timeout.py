@@ -7,8 +7,7 @@ run out.  The call then records SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT; the CTA
 that gave up drains its copies and MMAs, frees its tensor memory and exits,
 and the kernel completes well before the default 1 s limit.  The next normal
 call on the same workspace must read a clear error word and match the oracle
-(the GPU stays usable).  With the combine queue in use, warps waiting for
-queue slots that the starved item would have closed give up the same way.
+(the GPU stays usable).
 """
 import time
 
@@ -38,8 +37,8 @@ def tiny():
     return shape, w_gu, w_d, wr
 
 
-# (8, 2): every combine done inline by the down item that completes it;
-# (300, 8): B*k >= 32 m', the grid-wide combine queue is in use
+# (8, 2): one work entry per expert; (300, 8): two entries per expert, so
+# the starved item's entry shares its expert with a running one
 @pytest.mark.parametrize("B,k", [(8, 2), (300, 8)])
 def test_dependency_wait_runs_out_and_next_call_is_clean(tiny, B, k):
     shape, w_gu, w_d, wr = tiny
