@@ -568,7 +568,7 @@ def main_gpu(args, ws, rank, local):
         "step_ms_p10_p50_p90": [pt["step_ms_p10"], pt["step_ms_p50"], pt["step_ms_p90"]],
         "step_spread": "percentiles of the mean step over blocks of 10 consecutive layer calls",
         "graph": graph,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": 4 * args.steps,   # route, group, expert FFN, combine per step
         "clocks": clk.summary(),
     }
     if not args.no_pruned:
