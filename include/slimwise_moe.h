@@ -51,7 +51,7 @@ typedef enum slimwise_status {
 
 /* Device-side error bits reported by slimwise_moe_device_status(). */
 #define SLIMWISE_DEVERR_PIPELINE_TIMEOUT 0x1   /* an mbarrier wait gave up        */
-#define SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT 0x2 /* gate/up -> down, or combine-queue, wait gave up */
+#define SLIMWISE_DEVERR_DEPENDENCY_TIMEOUT 0x2 /* a down item's wait for its gate/up tiles gave up */
 #define SLIMWISE_DEVERR_DUPLICATE_RETAINED 0x4 /* retained_idx has a repeated id  */
 #define SLIMWISE_DEVERR_BAD_RETAINED 0x8       /* retained_idx has an id outside [0,E) */
 #define SLIMWISE_DEVERR_BAD_TOPK 0x10          /* a given top-k id outside [0,E)  */
@@ -117,9 +117,10 @@ int slimwise_moe_decode_full(const void *hidden, const float *router_w,
 /*
  * Launch options for slimwise_moe_decode_ex (all fields may be zero).
  *   ffn_begin / ffn_end  cudaEvent_t recorded on `stream` immediately before
- *                        and after the expert-FFN kernel (NULL: none); used to
- *                        time that kernel alone.
- *   disable_pdl          1: launch the three kernels with plain stream
+ *                        the expert-FFN kernel and after the combine kernel
+ *                        that follows it (NULL: none); used to time the two
+ *                        alone.
+ *   disable_pdl          1: launch the layer's four kernels with plain stream
  *                        ordering instead of programmatic dependent launch.
  *   grid_ctas            >0: persistent expert-FFN grid size (default: the
  *                        device's SM count).

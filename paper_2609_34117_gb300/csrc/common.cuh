@@ -194,7 +194,29 @@ struct Dims {
   int tok_chunk;  // max tokens of one expert per work item (multiple of 16, 16..256)
   int Is;         // shared-expert intermediate width (0: no shared expert)
   int S;          // shared-expert work entries: ceil(B / tok_chunk), 0 without one
+  int wide;       // 1: a routed work item covers two adjacent 128-row weight tiles
 };
+
+// Work items per entry: routed gate/up tiles (64 gate + 64 up rows each, or
+// twice that for wide items) and down tiles (128 rows of W_down, or 256).
+__host__ __device__ inline int gate_up_tiles(const Dims &d) {
+  return d.I / (kGateRows * (d.wide ? 2 : 1));
+}
+__host__ __device__ inline int down_tiles(const Dims &d) {
+  return d.H / (kTileRows * (d.wide ? 2 : 1));
+}
+// Wide items need whole 256-row tiles of both weights and no shared expert
+// (its items keep 128 rows, and a stage holds one kind of A tile).  Two
+// weight tiles then share each stage's token rows, which halves the token
+// rows read per weight byte, but a stage grows by 16 KB and an expert has
+// half as many items.  Measured on the Qwen-class layer, they pay at token
+// chunks of 64-80 rows with pools of 64 or more experts (the skewed 40-layer
+// stack 8 % faster, uniform B = 256 with m' = 64 faster); with larger chunks
+// too few stages fit, and with smaller pools too few items remain to balance
+// the SMs (B = 128 with m' = 32 was 15 % slower).
+constexpr int kWideMinChunk = 64;
+constexpr int kWideMaxChunk = 80;
+constexpr int kWideMinPool = 64;
 
 // Kernel launch declarations (defined in their own translation units).
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,

@@ -52,24 +52,21 @@ constexpr int kItemRing = 4;
 constexpr int kXchStride = 17;  // padded row stride (floats) of the exchange buffer
 constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
 
-// 64-wide K sub-tiles per pipeline stage (one 128-byte swizzle atom each).
-#ifndef SLIMWISE_STAGE_SUB
-#define SLIMWISE_STAGE_SUB 1
-#endif
-constexpr int kStageSub = SLIMWISE_STAGE_SUB;
-
+// A pipeline stage: one 64-wide K sub-tile (one 128-byte swizzle atom) of
+// the item's weight rows -- 128, or 256 for a wide item -- then tok_chunk
+// token rows of the same K range.
 struct FfnSmem {
   int stages;
+  int a_bytes;
   int stage_bytes;
-  int b_sub_bytes;
   size_t xch_off, bar_off, misc_off, total;
 };
 
-__host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
+__host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages, int wide) {
   FfnSmem p;
   p.stages = stages;
-  p.b_sub_bytes = tok_chunk * kBlockK * 2;
-  p.stage_bytes = kStageSub * (kATileBytes + p.b_sub_bytes);
+  p.a_bytes = kATileBytes * (wide ? 2 : 1);
+  p.stage_bytes = p.a_bytes + tok_chunk * kBlockK * 2;
   p.xch_off = (size_t)stages * p.stage_bytes;
   p.bar_off = p.xch_off + kXchBytes;
   // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
@@ -78,6 +75,11 @@ __host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages) {
   p.total = p.misc_off + 4 * (kItemRing + 3) + 1024;
   return p;
 }
+
+// TMEM accumulators: one per 128 weight rows of an item, N = tok_chunk
+// columns each, in two buffers (the epilogue of one item overlaps the MMAs
+// of the next): at most 512 columns, so wide items need tok_chunk <= 128.
+__host__ __device__ inline int ffn_acc_cols(const Dims &d) { return (d.wide ? 2 : 1) * d.tok_chunk; }
 
 struct Item {
   int down;      // 0: gate/up, 1: down
@@ -227,7 +229,7 @@ __device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit
 // At most 128 registers a thread (320 threads: 40 K of the SM's 64 K), so
 // that a CTA of the dependent combine kernel (256 threads, 72 registers)
 // can become resident beside this one.
-template <bool kShared>
+template <bool kShared, bool kWide>
 __global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out, int stages,
@@ -237,7 +239,7 @@ __global__ void __maxnreg__(128)
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const FfnSmem plan = ffn_smem_plan(d.tok_chunk, stages);
+  const FfnSmem plan = ffn_smem_plan(d.tok_chunk, stages, d.wide);
   const uint32_t smem_base = smem_u32(smem);
   float *xch = reinterpret_cast<float *>(smem + plan.xch_off);
   const uint32_t bar0 = smem_base + (uint32_t)plan.bar_off;
@@ -306,17 +308,19 @@ __global__ void __maxnreg__(128)
   // so a wrong guess costs bandwidth, never correctness.
   if constexpr (!kShared) {
     if (warp == 0 && lane == 0) {
-      const int t1g = d.I / kGateRows;
+      const int t1g = gate_up_tiles(d);
+      const int rows = kGateRows * (d.wide ? 2 : 1);  // gate rows (and up rows) of a tile
       const int entry = blockIdx.x / t1g;
       const int n_prev = __ldcg(&ws.ctrl[kCtrlNumEntries]);
       if (entry < n_prev && entry < max_entries_for(d.B, d.E, d.k, d.Is)) {
         const int e = __ldcg(&ws.entries[entry]).x;
         if (e >= 0 && e < d.E) {
-          const int row0 = e * 2 * d.I + (blockIdx.x - entry * t1g) * kGateRows;
-          for (int kc = 0; kc < d.H / kBlockK; ++kc) {
-            tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0);
-            tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + d.I);
-          }
+          const int row0 = e * 2 * d.I + (blockIdx.x - entry * t1g) * rows;
+          for (int r = 0; r < rows; r += kGateRows)
+            for (int kc = 0; kc < d.H / kBlockK; ++kc) {
+              tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + r);
+              tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + d.I + r);
+            }
         }
       }
     }
@@ -335,15 +339,16 @@ __global__ void __maxnreg__(128)
 #endif
 
   const int total = __ldcg(&ws.ctrl[kCtrlTotalItems]);
-  const int t1 = d.I / kGateRows;
-  const int t2 = d.H / kTileRows;
+  const int t1 = gate_up_tiles(d);
+  const int t2 = down_tiles(d);
   ItemPlan ip;
   ip.r1 = __ldcg(&ws.ctrl[kCtrlItems1]);
   ip.t1 = t1;
   ip.t1s = kShared ? d.Is / kGateRows : 0;
   ip.t2 = t2;
   ip.S = kShared ? d.S : 0;
-  const int nb_cols = d.tok_chunk;  // TMEM columns per accumulator buffer
+  const int nb_cols = ffn_acc_cols(d);  // TMEM columns per accumulator buffer
+  constexpr int wmul = kWide ? 2 : 1;   // 128-row halves of a routed item
 
 
   if (warp == 0) {
@@ -408,30 +413,34 @@ __global__ void __maxnreg__(128)
         // the item's token rows: one box of the tokens rounded up to 16
         // rows (rows past the entry are loaded but not multiplied)
         const int box_m = token_box_for(it.n16);
-        int nsub_total, row0, row1;
+        // weight rows: per 128-row half of the item, two 64-row boxes -- the
+        // gate rows and the matching up rows, or 128 consecutive down rows
+        const int halves = (kShared && it.shared) ? 1 : wmul;
+        const int hstep = it.down ? kTileRows : kGateRows;  // row offset of half 1
+        int nk, row0, row1;
         const void *amap;
         const void *bmap;
         if (kShared && it.shared) {
           // the shared expert: its own weights, tokens in batch order
-          nsub_total = it.down ? d.Is / kBlockK : d.H / kBlockK;
+          nk = it.down ? d.Is / kBlockK : d.H / kBlockK;
           amap = it.down ? (const void *)&maps.w_down_s : (const void *)&maps.w_gu_s;
           bmap = it.down ? (const void *)&maps.act_s[box_m] : (const void *)&maps.xt[box_m];
           row0 = it.down ? it.tile * kTileRows : it.tile * kGateRows;
           row1 = it.down ? row0 + kGateRows : row0 + d.Is;
         } else {
-          nsub_total = it.down ? d.I / kBlockK : d.H / kBlockK;
+          nk = it.down ? d.I / kBlockK : d.H / kBlockK;
           amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
           bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
           if (it.down) {
-            row0 = it.expert * d.H + it.tile * kTileRows;
+            row0 = it.expert * d.H + it.tile * kTileRows * halves;
             row1 = row0 + kGateRows;
           } else {
-            row0 = it.expert * 2 * d.I + it.tile * kGateRows;
+            row0 = it.expert * 2 * d.I + it.tile * kGateRows * halves;
             row1 = row0 + d.I;
           }
         }
-        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
-        const uint32_t sub_bytes = (uint32_t)(kATileBytes + kTokBox * (box_m + 1) * kBlockK * 2);
+        const uint32_t stage_tx =
+            (uint32_t)(halves * kATileBytes + kTokBox * (box_m + 1) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, timeout_ns)) {
@@ -439,18 +448,15 @@ __global__ void __maxnreg__(128)
             ok = false;
             break;
           }
-          const int nsub = min(kStageSub, nsub_total - kc * kStageSub);
+          const int x = kc * kBlockK;
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
-          const uint32_t b = a + kStageSub * kATileBytes;
-          mbar_arrive_expect_tx(full_bar(stage), nsub * sub_bytes);
-          for (int s = 0; s < nsub; ++s) {
-            const int x = (kc * kStageSub + s) * kBlockK;
-            const uint32_t as = a + s * kATileBytes;
-            const uint32_t bs = b + s * (uint32_t)plan.b_sub_bytes;
-            tma_load_2d(as, amap, full_bar(stage), x, row0, pol_w);
-            tma_load_2d(as + kATileBytes / 2, amap, full_bar(stage), x, row1, pol_w);
-            tma_load_2d(bs, bmap, full_bar(stage), x, it.slot_base, pol_x);
+          mbar_arrive_expect_tx(full_bar(stage), stage_tx);
+          for (int h = 0; h < halves; ++h) {
+            const uint32_t ah = a + (uint32_t)(h * kATileBytes);
+            tma_load_2d(ah, amap, full_bar(stage), x, row0 + h * hstep, pol_w);
+            tma_load_2d(ah + kATileBytes / 2, amap, full_bar(stage), x, row1 + h * hstep, pol_w);
           }
+          tma_load_2d(a + (uint32_t)plan.a_bytes, bmap, full_bar(stage), x, it.slot_base, pol_x);
           ++issued;
           if (++stage == stages) {
             stage = 0;
@@ -495,11 +501,13 @@ __global__ void __maxnreg__(128)
           break;
         }
         tc_fence_after();
+        // half h of the item: A = the stage's weight rows [128 h, 128 h + 128),
+        // D = columns [h tok_chunk, ...) of the buffer; B = the token rows
         const uint32_t d_tmem = tmem_base + (uint32_t)(b * nb_cols);
         const uint32_t idesc = idesc_bf16_f32(kTileRows, it.n16 * kTokBox);
+        const int halves = (kShared && it.shared) ? 1 : wmul;
         const int inner = (kShared && it.shared) ? d.Is : d.I;
-        const int nsub_total = it.down ? inner / kBlockK : d.H / kBlockK;
-        const int nk = (nsub_total + kStageSub - 1) / kStageSub;
+        const int nk = it.down ? inner / kBlockK : d.H / kBlockK;
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(full_bar(stage), phase, abort, timeout_ns)) {
@@ -511,17 +519,14 @@ __global__ void __maxnreg__(128)
 #ifdef SLIMWISE_TRACE
           if (blockIdx.x == 0 && n_consumed == 0) trace_stamp(ws, tr_step, kTrFfnFirstData);
 #endif
-          const int nsub = min(kStageSub, nsub_total - kc * kStageSub);
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
-          const uint32_t b = a + kStageSub * kATileBytes;
-          for (int s = 0; s < nsub; ++s) {
-            const uint32_t as = a + s * kATileBytes;
-            const uint32_t bs = b + s * (uint32_t)plan.b_sub_bytes;
+          const uint32_t bs = a + (uint32_t)plan.a_bytes;
+          for (int h = 0; h < halves; ++h) {
+            const uint32_t as = a + (uint32_t)(h * kATileBytes);
 #pragma unroll
             for (int kk = 0; kk < kBlockK / 16; ++kk)
-              tc_mma_bf16(d_tmem, smem_desc_sw128(as + kk * 32),
-                          smem_desc_sw128(bs + kk * 32), idesc,
-                          (kc | s | kk) != 0 ? 1u : 0u);
+              tc_mma_bf16(d_tmem + (uint32_t)(h * d.tok_chunk), smem_desc_sw128(as + kk * 32),
+                          smem_desc_sw128(bs + kk * 32), idesc, (kc | kk) != 0 ? 1u : 0u);
           }
           tc_commit(empty_bar(stage));
           issued_any = true;
@@ -567,6 +572,7 @@ __global__ void __maxnreg__(128)
       if (b != g) continue;
       const Item it = decode_item<kShared>(item, ip, ws);
       const uint32_t use = (uint32_t)(local >> 1);
+      const int halves = (kShared && it.shared) ? 1 : wmul;
       got = mbar_wait_bounded(accf_bar(b), use & 1u, abort, timeout_ns);
       if (!got && !*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
       if (!epi_all(g, got)) break;
@@ -576,37 +582,41 @@ __global__ void __maxnreg__(128)
         // gate rows live in TMEM lanes 0..63, the matching up rows in 64..127
         const int n_loc = et >> 3;          // token column within a 16-chunk
         const int i0 = (et & 7) * 8;        // 8 consecutive intermediate indices
-        for (int c = 0; c < it.n16; ++c) {
-          uint32_t v[16];
-          tmem_ld16(taddr + c * 16, v);
-          tmem_ld_wait();
+        for (int hh = 0; hh < halves; ++hh) {
+          // half hh of a wide item is the 64 gate + 64 up rows of tile 2 t + hh
+          const int act_col = (it.tile * halves + hh) * kGateRows + i0;
+          for (int c = 0; c < it.n16; ++c) {
+            uint32_t v[16];
+            tmem_ld16(taddr + (uint32_t)(hh * d.tok_chunk) + c * 16, v);
+            tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 16; ++j) xb[row * kXchStride + j] = __uint_as_float(v[j]);
-          epi_bar(g);
-          const int col = c * 16 + n_loc;
-          if (col < it.n) {
-            uint32_t packed[4];
+            for (int j = 0; j < 16; ++j) xb[row * kXchStride + j] = __uint_as_float(v[j]);
+            epi_bar(g);
+            const int col = c * 16 + n_loc;
+            if (col < it.n) {
+              uint32_t packed[4];
 #pragma unroll
-            for (int ii = 0; ii < 8; ii += 2) {
-              float a2[2];
+              for (int ii = 0; ii < 8; ii += 2) {
+                float a2[2];
 #pragma unroll
-              for (int u2 = 0; u2 < 2; ++u2) {
-                const float gv = xb[(i0 + ii + u2) * kXchStride + n_loc];
-                const float uv = xb[(kGateRows + i0 + ii + u2) * kXchStride + n_loc];
-                // SiLU(g) * u = g / (1 + e^-g) * u
-                a2[u2] = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
+                for (int u2 = 0; u2 < 2; ++u2) {
+                  const float gv = xb[(i0 + ii + u2) * kXchStride + n_loc];
+                  const float uv = xb[(kGateRows + i0 + ii + u2) * kXchStride + n_loc];
+                  // SiLU(g) * u = g / (1 + e^-g) * u
+                  a2[u2] = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
+                }
+                __nv_bfloat162 h2 = __floats2bfloat162_rn(a2[0], a2[1]);
+                packed[ii / 2] = *reinterpret_cast<uint32_t *>(&h2);
               }
-              __nv_bfloat162 h2 = __floats2bfloat162_rn(a2[0], a2[1]);
-              packed[ii / 2] = *reinterpret_cast<uint32_t *>(&h2);
+              // routed: grouped order [B*k, I]; shared: token order [B, Is]
+              __nv_bfloat16 *arow = (kShared && it.shared)
+                                        ? ws.act_s + (size_t)(it.slot_base + col) * d.Is
+                                        : ws.act + (size_t)(it.slot_base + col) * d.I;
+              *reinterpret_cast<uint4 *>(arow + act_col) =
+                  make_uint4(packed[0], packed[1], packed[2], packed[3]);
             }
-            // routed: grouped order [B*k, I]; shared: token order [B, Is]
-            __nv_bfloat16 *arow = (kShared && it.shared)
-                                      ? ws.act_s + (size_t)(it.slot_base + col) * d.Is
-                                      : ws.act + (size_t)(it.slot_base + col) * d.I;
-            *reinterpret_cast<uint4 *>(arow + it.tile * kGateRows + i0) =
-                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+            epi_bar(g);  // the exchange buffer is rewritten by the next chunk
           }
-          epi_bar(g);  // the exchange buffer is rewritten by the next chunk
         }
         tc_fence_before();
         mbar_arrive(acce_bar(b));
@@ -616,17 +626,19 @@ __global__ void __maxnreg__(128)
         epi_bar(g);
         if (et == 0) atomicAdd(&ws.entry_done[it.entry], 1);
       } else {
-        const int h = it.tile * kTileRows + row;
         float *ybase = (kShared && it.shared) ? ws.y_s : ws.y;  // token / grouped order
-        for (int c = 0; c < it.n16; ++c) {
-          uint32_t v[16];
-          tmem_ld16(taddr + c * 16, v);
-          tmem_ld_wait();
+        for (int hh = 0; hh < halves; ++hh) {
+          const int h = (it.tile * halves + hh) * kTileRows + row;
+          for (int c = 0; c < it.n16; ++c) {
+            uint32_t v[16];
+            tmem_ld16(taddr + (uint32_t)(hh * d.tok_chunk) + c * 16, v);
+            tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int col = c * 16 + j;
-            if (col < it.n)
-              ybase[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
+            for (int j = 0; j < 16; ++j) {
+              const int col = c * 16 + j;
+              if (col < it.n)
+                ybase[(size_t)(it.slot_base + col) * d.H + h] = __uint_as_float(v[j]);
+            }
           }
         }
         // the expert outputs are all a down item writes: the combine kernel
@@ -691,9 +703,9 @@ cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStre
   return cudaLaunchKernelEx(&cfg, combine_kernel<false>, d, ws, out);
 }
 
-int ffn_stages_for(int tok_chunk, size_t smem_limit) {
+int ffn_stages_for(int tok_chunk, int wide, size_t smem_limit) {
   int s = 12;
-  while (s > 2 && ffn_smem_plan(tok_chunk, s).total + 1024 > smem_limit) --s;
+  while (s > 2 && ffn_smem_plan(tok_chunk, s, wide).total + 1024 > smem_limit) --s;
   return s;
 }
 
@@ -716,14 +728,20 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
     return cudaErrorInvalidValue;
   // the dependent combine kernel needs no shared memory: every byte the
   // block may opt into goes to pipeline stages
-  const int stages = ffn_stages_for(d.tok_chunk, (size_t)optin);
-  const size_t smem = ffn_smem_plan(d.tok_chunk, stages).total + 1024;
+  const int stages = ffn_stages_for(d.tok_chunk, d.wide, (size_t)optin);
+  const size_t smem = ffn_smem_plan(d.tok_chunk, stages, d.wide).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
-  auto kernel = d.Is > 0 ? expert_ffn_kernel<true> : expert_ffn_kernel<false>;
+  // wide items only without a shared expert, on whole 256-row tiles, with
+  // both accumulators of two buffers in the 512 TMEM columns
+  if (d.wide && (d.Is > 0 || d.I % (2 * kGateRows) != 0 || d.H % (2 * kTileRows) != 0 ||
+                 d.tok_chunk > 128))
+    return cudaErrorInvalidValue;
+  auto kernel = d.Is > 0 ? expert_ffn_kernel<true, false>
+                         : d.wide ? expert_ffn_kernel<false, true> : expert_ffn_kernel<false, false>;
   err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
   int tmem_cols = 32;
-  while (tmem_cols < 2 * d.tok_chunk) tmem_cols <<= 1;
+  while (tmem_cols < 2 * ffn_acc_cols(d)) tmem_cols <<= 1;
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);

@@ -234,8 +234,8 @@ __global__ void __launch_bounds__(kGroupThreads)
     ws.entries[sidx] = make_int4(-1, sidx * d.tok_chunk, min(d.tok_chunk, B - sidx * d.tok_chunk), 0);
   for (int i = gtid; i < n_se + n_entries; i += gstride) ws.entry_done[i] = 0;
   if (blockIdx.x == 0 && tid == 0) {
-    const int t1_items = d.I / kGateRows;
-    const int t2_items = d.H / kTileRows;
+    const int t1_items = gate_up_tiles(d);
+    const int t2_items = down_tiles(d);
     const int t1s_items = d.Is / kGateRows;
     ws.offsets[E] = offs[E];
     ws.ctrl[kCtrlUnionSize] = U;

@@ -106,6 +106,9 @@ Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret, int32_
   }
   d.Is = Is;
   d.S = Is > 0 ? (d.B + d.tok_chunk - 1) / d.tok_chunk : 0;
+  d.wide = (Is == 0 && d.I % (2 * kGateRows) == 0 && d.H % (2 * kTileRows) == 0 &&
+            d.tok_chunk >= kWideMinChunk && d.tok_chunk <= kWideMaxChunk &&
+            m_ret >= kWideMinPool) ? 1 : 0;
   return d;
 }
 

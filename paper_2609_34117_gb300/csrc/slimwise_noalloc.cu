@@ -5,7 +5,7 @@
 // routine during inference: a serving engine that sized and carved out all
 // of its device memory up front, code that runs under a memory pool or
 // allocator it does not control, or a plugin given only its inputs and
-// outputs.  slimwise_moe_decode_noalloc serves them by running the same three
+// outputs.  slimwise_moe_decode_noalloc serves them by running the same four
 // kernels as slimwise_moe_decode with the scratch memory (routing state,
 // grouped activations, expert outputs, counters) placed in a fixed device
 // array that belongs to this library.

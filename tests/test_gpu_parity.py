@@ -300,6 +300,22 @@ def test_hot_expert_spans_several_slots(B, m_prime, hot):
     assert route["counts"].max() == B
 
 
+@pytest.mark.parametrize("B,skew", [(256, False), (256, True), (200, False)])
+def test_wide_items_every_output(B, skew):
+    # 64 of 128 experts, top-8: a mean load of 32 (25 at B = 200) gives token
+    # chunks of 64 rows, where each work item covers two adjacent 128-row
+    # weight tiles sharing each stage's token rows (two accumulators per
+    # item).  Every output and the whole routing against the oracle, with
+    # uniform and Zipf-skewed routing (popular experts in several entries).
+    shape = synth.LayerShape(hidden=256, num_experts=128, inter=256, top_k=8)
+    layer = Layer(shape, seed=19)
+    x, wr = synth.hidden_states(B, shape, 160 + B), None
+    if skew:
+        bias = synth.zipf_rank_bias(shape.num_experts, 1.1, 161)
+        x, wr = synth.apply_popularity_bias(x, layer.wr, bias)
+    _case(layer, B=B, m_prime=64, seed_x=160 + B, seed_imp=21, x=x, wr=wr)
+
+
 @pytest.mark.parametrize("B", [1, 5, 17, 33, 300])
 def test_ragged_batches_and_token_chunks(tiny, B):
     # k = m' = 8: every token selects every retained expert, so each expert
