@@ -232,12 +232,17 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   __syncthreads();
 
   // Logits of this CTA's slice [r_lo, r_hi) of the retained list.  With at
-  // least two rows per warp, a warp takes its rows in pairs (rows r, r + 1),
-  // which halves the shared-memory reads of the staged hidden rows; the sums
-  // and their order are those of one row at a time.
+  // least two rows per warp (at 8 tokens per cluster: two rows per slice), a
+  // warp takes its rows in pairs (rows r, r + 1), which halves the
+  // shared-memory reads of the staged hidden rows; the sums and their order
+  // are those of one row at a time.
   const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
   const int nchunks = H / 128;
-  const int npair = (r_hi - r_lo >= 2 * kRouteWarps) ? (r_hi - r_lo) / 2 : 0;
+  // At 8 tokens per cluster the staged rows' shared-memory reads bound the
+  // logits, so pairs pay from two rows on (1.6 us at B = 256, m' = 64); at
+  // 16 tokens (fewer warps busy) they lost 2 us at B = 512, m' = 32.
+  const int npair = ((TB == 8 && r_hi - r_lo >= 2) || r_hi - r_lo >= 2 * kRouteWarps)
+                        ? (r_hi - r_lo) / 2 : 0;
   for (int pi = warp; pi < npair; pi += kRouteWarps) {
     const int r = r_lo + 2 * pi;
     const float4 *w0 = reinterpret_cast<const float4 *>(router_w + (size_t)ids[r] * H) + lane;
