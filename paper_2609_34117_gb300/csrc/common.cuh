@@ -244,8 +244,10 @@ constexpr uint64_t kDefaultWaitLimitNs = 1000000000ull;
 // The gate-weighted combine of every (token, 128-column tile), after the
 // expert FFN.
 cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStream_t stream);
+// retained: the call's retained ids (NULL: the full pool or a compacted one),
+// read only to guess which weight tiles to warm in L2.
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
-                              __nv_bfloat16 *out, int grid, bool pdl,
+                              __nv_bfloat16 *out, const int32_t *retained, int grid, bool pdl,
                               cudaStream_t stream, uint64_t timeout_ns = kDefaultWaitLimitNs,
                               int starve_first_down = 0);
 

@@ -268,7 +268,7 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
                                   ? (uint64_t)opts->wait_limit_ns
                                   : kDefaultWaitLimitNs;
   const int starve = (opts && opts->test_starve_first_down) ? 1 : 0;
-  if (launch_expert_ffn(maps, d, w, static_cast<__nv_bfloat16 *>(out), grid,
+  if (launch_expert_ffn(maps, d, w, static_cast<__nv_bfloat16 *>(out), retained, grid,
                         pdl && !timed, st, wait_limit, starve) != cudaSuccess)
     return SLIMWISE_ERR_CUDA;
   // the combine belongs to the timed span: the events bracket the expert FFN
