@@ -131,12 +131,12 @@ inline WsLayout make_layout(int B, int H, int E, int I, int k, int Is = 0) {
   L.pos = take(slots * 4);
   L.xp = take(slots * H * 2);
   L.act = take(slots * I * 2);
-  L.y = take(slots * H * 4);
+  L.y = take(slots * H * 2);
   if (Is > 0) {
     L.shared_gate = take((size_t)B * 4);
     L.xt = take((size_t)B * H * 2);
     L.act_s = take((size_t)B * Is * 2);
-    L.y_s = take((size_t)B * H * 4);
+    L.y_s = take((size_t)B * H * 2);
   } else {  // no shared expert: no space (these regions are never accessed)
     L.shared_gate = L.xt = L.act_s = L.y_s = o;
   }
@@ -158,11 +158,11 @@ struct Ws {
   int32_t *pos;
   __nv_bfloat16 *xp;   // [B*k, H] hidden rows in grouped order
   __nv_bfloat16 *act;  // [B*k, I] SwiGLU activations in grouped order
-  float *y;            // [B*k, H] expert outputs in grouped order
+  __nv_bfloat16 *y;    // [B*k, H] expert outputs in grouped order
   float *shared_gate;  // [B] sigmoid gate of the shared expert
   __nv_bfloat16 *xt;   // [B, H] hidden rows, token order (shared-expert input)
   __nv_bfloat16 *act_s;  // [B, Is] shared-expert activations, token order
-  float *y_s;          // [B, H] shared-expert outputs, token order
+  __nv_bfloat16 *y_s;  // [B, H] shared-expert outputs, token order
 };
 
 inline Ws make_ws(void *base, const WsLayout &L) {
@@ -180,11 +180,11 @@ inline Ws make_ws(void *base, const WsLayout &L) {
   w.pos = (int32_t *)(b + L.pos);
   w.xp = (__nv_bfloat16 *)(b + L.xp);
   w.act = (__nv_bfloat16 *)(b + L.act);
-  w.y = (float *)(b + L.y);
+  w.y = (__nv_bfloat16 *)(b + L.y);
   w.shared_gate = (float *)(b + L.shared_gate);
   w.xt = (__nv_bfloat16 *)(b + L.xt);
   w.act_s = (__nv_bfloat16 *)(b + L.act_s);
-  w.y_s = (float *)(b + L.y_s);
+  w.y_s = (__nv_bfloat16 *)(b + L.y_s);
   return w;
 }
 

@@ -3,8 +3,8 @@
 //
 // The statistics are taken from a full-pool layer call: its workspace holds,
 // for every (token, selection) slot in grouped order (expert ascending, token
-// ascending), the selected expert's fp32 output row y and, through perm, the
-// slot's gate.  For each expert e and each token t routed to it:
+// ascending), the selected expert's output row y (accumulated in fp32, stored
+// as bf16) and, through perm, the slot's gate.  For each expert e and each token t routed to it:
 //   stats[e][0] += 1             tokens routed to e
 //   stats[e][1] += g_te          routing mass
 //   stats[e][2] += ||y||_2       expert activation norm (EAN)
@@ -25,16 +25,19 @@ __global__ void __launch_bounds__(kStatsWarps * 32)
   const int p0 = __ldcg(&ws.offsets[e]), p1 = __ldcg(&ws.offsets[e + 1]);
   double cnt = 0.0, mass = 0.0, ean = 0.0, reap = 0.0;
   for (int p = p0; p < p1; ++p) {
-    // ||y||^2: lane l sums its 4-wide columns 128c + 4l .. +3, then an xor
+    // ||y||^2: lane l sums its 8-wide columns 256c + 8l .. +7, then an xor
     // butterfly over the lanes
-    const float4 *row = reinterpret_cast<const float4 *>(ws.y + (size_t)p * d.H);
+    const uint4 *row = reinterpret_cast<const uint4 *>(ws.y + (size_t)p * d.H);
     float s = 0.0f;
-    for (int c = lane; c < d.H / 4; c += 32) {
-      const float4 v = __ldcg(row + c);
-      s = fmaf(v.x, v.x, s);
-      s = fmaf(v.y, v.y, s);
-      s = fmaf(v.z, v.z, s);
-      s = fmaf(v.w, v.w, s);
+    for (int c = lane; c < d.H / 8; c += 32) {
+      const uint4 v = __ldcg(row + c);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float a = __uint_as_float(w[q] << 16), b = __uint_as_float(w[q] & 0xFFFF0000u);
+        s = fmaf(a, a, s);
+        s = fmaf(b, b, s);
+      }
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, off);

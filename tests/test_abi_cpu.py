@@ -47,8 +47,8 @@ def test_workspace_size_grows_with_batch_and_covers_buffers(lib):
     prev = 0
     for B in (1, 8, 64, 256, 512):
         n = _ws(B, H, E, I, k)
-        # grouped hidden rows (bf16), activations (bf16) and expert outputs (fp32)
-        assert n >= B * k * (2 * H + 2 * I + 4 * H)
+        # grouped hidden rows, activations and expert outputs (all bf16)
+        assert n >= B * k * (2 * H + 2 * I + 2 * H)
         assert n > prev
         prev = n
     assert _ws(0, H, E, I, k) > 0
@@ -128,7 +128,7 @@ def test_shared_expert_entry_points_validate_without_cuda(lib):
     # rows, activations and outputs
     n0 = _ws(64, 2048, 128, 768, 8)
     assert lib.slimwise_moe_shared_workspace_size(ctypes.byref(s64), 8, 1024, ctypes.byref(out)) == 0
-    assert out.value >= n0 + 64 * (4 + 2 * 2048 + 2 * 1024 + 4 * 2048)
+    assert out.value >= n0 + 64 * (4 + 2 * 2048 + 2 * 1024 + 2 * 2048)
     s = binding.Shape(4, 256, 16, 128)
     for bad_is in (0, 32, 96, 1 << 17):
         assert lib.slimwise_moe_shared_workspace_size(ctypes.byref(s), 2, bad_is, ctypes.byref(out)) == 2
