@@ -153,14 +153,8 @@ __device__ __forceinline__ Item decode_item(int item, const ItemPlan &ip, const 
 template <bool kShared>
 __device__ __forceinline__ void combine_token(const Ws &ws, const Dims &d,
                                               __nv_bfloat16 *__restrict__ out, int t, int tile,
-                                              int lane) {
+                                              int lane, int p, float gj, float sg) {
   const __nv_bfloat16 *ytile = ws.y + tile * kCombineTile + 4 * lane;
-  int p = 0;
-  float gj = 0.0f;
-  if (lane < d.k) {
-    p = __ldcg(&ws.pos[(size_t)t * d.k + lane]);
-    gj = __ldcg(&ws.topk_gate[(size_t)t * d.k + lane]);
-  }
   float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   for (int j0 = 0; j0 < d.k; j0 += 8) {
     uint2 v[8];
@@ -183,7 +177,6 @@ __device__ __forceinline__ void combine_token(const Ws &ws, const Dims &d,
   }
   if constexpr (kShared) {
     // the shared expert's term, after the k routed ones (Sec. 3.3)
-    const float sg = __ldcg(&ws.shared_gate[t]);
     const uint2 vs = __ldcg(reinterpret_cast<const uint2 *>(
         ws.y_s + (size_t)t * d.H + tile * kCombineTile + 4 * lane));
     acc.x = fmaf(sg, __uint_as_float(vs.x << 16), acc.x);
@@ -683,15 +676,31 @@ constexpr int kCombineThreads = 256;
 template <bool kShared>
 __global__ void __launch_bounds__(kCombineThreads)
     combine_kernel(Dims d, Ws ws, __nv_bfloat16 *__restrict__ out) {
-  pdl_wait_primary();
-  // the next call's routing may become resident; it waits for this grid
-  pdl_launch_dependents();
   const int t2 = d.H / kCombineTile;
   const int lane = threadIdx.x & 31;
   const int wpc = kCombineThreads / 32;
   const int pairs = d.B * t2;
-  for (int p = blockIdx.x * wpc + (threadIdx.x >> 5); p < pairs; p += gridDim.x * wpc)
-    combine_token<kShared>(ws, d, out, p / t2, p - (p / t2) * t2, lane);
+  // One pair per warp (the grid covers them all).  Its grouped positions and
+  // gates were written by the routing and grouping kernels, which finished
+  // before the expert FFN started its work, so they are read before waiting
+  // for the FFN; only the expert outputs need the wait.
+  const int pr = blockIdx.x * wpc + (threadIdx.x >> 5);
+  const int t = pr / t2;
+  int p = 0;
+  float gj = 0.0f, sg = 0.0f;
+  if (pr < pairs) {
+    if (lane < d.k) {
+      p = __ldcg(&ws.pos[(size_t)t * d.k + lane]);
+      gj = __ldcg(&ws.topk_gate[(size_t)t * d.k + lane]);
+    }
+    if constexpr (kShared) sg = __ldcg(&ws.shared_gate[t]);
+  }
+  pdl_wait_primary();
+  // The next call's routing is not signalled early: its CTAs would compete
+  // for SMs with this grid's (and, with 8-token routing clusters, wait for
+  // whole GPCs), which cost up to 7 us at B = 288, m' = 32.  It starts when
+  // this grid ends.
+  if (pr < pairs) combine_token<kShared>(ws, d, out, t, pr - t * t2, lane, p, gj, sg);
 }
 
 cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStream_t stream) {
