@@ -209,7 +209,7 @@ class LayerInputs:
         k = self.shape.top_k
         if self.shared is None:
             sw.slimwise_moe_decode_ex(x, self.wr, retained, w_gu, w_d, k, out=out, workspace=ws_buf,
-                                      stream=stream, ffn_events=ffn_events)
+                                      stream=stream, ffn_events=ffn_events, ffn_items=FFN_ITEMS)
         else:
             sw.slimwise_moe_decode_shared(x, self.wr, retained, w_gu, w_d, k, *self.shared, out=out,
                                           workspace=ws_buf, stream=stream, ffn_events=ffn_events)
@@ -571,6 +571,8 @@ def main_gpu(args, ws, rank, local):
         "gpu_launches": 4 * args.steps,   # route, group, expert FFN, combine per step
         "clocks": clk.summary(),
     }
+    if FFN_ITEMS:
+        result["ffn_items"] = FFN_ITEMS
     if not args.no_pruned:
         result["pruned"] = run_pruned(sw, device, peak, local)
     if args.sweep:
@@ -590,6 +592,10 @@ def main_gpu(args, ws, rank, local):
 
 
 PRUNED_POINTS = ("qwen_p50_b64", "qwen_p50_b256", "qwen_p75_b64")
+
+# form of the expert-FFN work items for the routed layers (--ffn-items; the
+# C ABI's slimwise_decode_opts.ffn_items: 0 the default, 1 CTA-pair items)
+FFN_ITEMS = 0
 
 
 def run_pruned(sw, device, peak, local, steps=4000):
@@ -823,9 +829,13 @@ def main():
     ap.add_argument("--stack40", action="store_true",
                     help="40 independent skewed layers at m'=64, B=256 (adds 'stack40')")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ffn-items", type=int, default=0, choices=[-1, 0, 1],
+                    help="expert-FFN work items: 0 default, 1 CTA-pair items")
     ap.add_argument("--no-pruned", action="store_true",
                     help="skip the pruned-layer points (adds 'pruned' by default)")
     args = ap.parse_args()
+    global FFN_ITEMS
+    FFN_ITEMS = args.ffn_items
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     ws, rank, local = dist_init()

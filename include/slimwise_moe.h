@@ -55,6 +55,7 @@ typedef enum slimwise_status {
 #define SLIMWISE_DEVERR_DUPLICATE_RETAINED 0x4 /* retained_idx has a repeated id  */
 #define SLIMWISE_DEVERR_BAD_RETAINED 0x8       /* retained_idx has an id outside [0,E) */
 #define SLIMWISE_DEVERR_BAD_TOPK 0x10          /* a given top-k id outside [0,E)  */
+#define SLIMWISE_DEVERR_TMEM_PAIR 0x20         /* the two CTAs of an FFN pair hold different tensor memory */
 
 /* Problem shape.  Supported: 0 <= B <= 2^20; H a multiple of 128 in
  * [128, 32768]; I a multiple of 64 in [64, 65536]; 1 <= E <= 1024.  Others
@@ -133,6 +134,15 @@ int slimwise_moe_decode_full(const void *hidden, const float *router_w,
  *   test_starve_first_down  tests only: 1 makes the first routed down item
  *                        wait for one more gate/up tile than exists, so that
  *                        wait runs out after wait_limit_ns (the timeout path).
+ *   ffn_items            form of the expert-FFN work items: 0 or -1 the
+ *                        default, 128-row items (256-row ones at token chunks
+ *                        of 64-80 rows); 1 CTA-pair items (two 128-row weight
+ *                        tiles on the two CTAs of a cluster, one M = 256
+ *                        tcgen05 MMA over both) wherever the layer allows
+ *                        them (no shared expert, H a multiple of 256, I of
+ *                        128).  The outputs agree within the layer's float
+ *                        tolerance in every form; pair items measured slower
+ *                        on the Qwen-class layer.
  */
 typedef struct slimwise_decode_opts {
   void *ffn_begin;
@@ -141,7 +151,7 @@ typedef struct slimwise_decode_opts {
   int32_t grid_ctas;
   int64_t wait_limit_ns;
   int32_t test_starve_first_down;
-  int32_t reserved;
+  int32_t ffn_items;
 } slimwise_decode_opts;
 
 /* slimwise_moe_decode with launch options; retained_idx NULL = full pool. */

@@ -27,6 +27,7 @@ DEVERR_DEPENDENCY_TIMEOUT = 0x2
 DEVERR_DUPLICATE_RETAINED = 0x4
 DEVERR_BAD_RETAINED = 0x8
 DEVERR_BAD_TOPK = 0x10
+DEVERR_TMEM_PAIR = 0x20
 
 EXPORTED = (
     "slimwise_status_string", "slimwise_moe_workspace_size", "slimwise_moe_decode",
@@ -53,7 +54,7 @@ class DecodeOpts(ctypes.Structure):
     _fields_ = [("ffn_begin", ctypes.c_void_p), ("ffn_end", ctypes.c_void_p),
                 ("disable_pdl", ctypes.c_int32), ("grid_ctas", ctypes.c_int32),
                 ("wait_limit_ns", ctypes.c_int64), ("test_starve_first_down", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("ffn_items", ctypes.c_int32)]
 
 
 def library_path() -> str:
@@ -258,9 +259,10 @@ def slimwise_moe_select_retained(stats, n_retained, criterion="reap", stream=Non
     return ids
 
 
-def _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns=0, test_starve_first_down=False):
+def _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns=0, test_starve_first_down=False,
+          ffn_items=0):
     opts = DecodeOpts(None, None, int(bool(disable_pdl)), int(grid_ctas), int(wait_limit_ns),
-                      int(bool(test_starve_first_down)), 0)
+                      int(bool(test_starve_first_down)), int(ffn_items))
     if ffn_events is not None:
         opts.ffn_begin = ctypes.c_void_p(ffn_events[0].cuda_event)
         opts.ffn_end = ctypes.c_void_p(ffn_events[1].cuda_event)
@@ -270,18 +272,20 @@ def _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns=0, test_starve_first
 def slimwise_moe_decode_ex(hidden, router_w, retained_idx, w_gate_up, w_down, top_k,
                            out=None, workspace=None, stream=None, ffn_events=None,
                            disable_pdl=False, grid_ctas=0, wait_limit_ns=0,
-                           test_starve_first_down=False):
+                           test_starve_first_down=False, ffn_items=0):
     """slimwise_moe_decode with launch options; retained_idx None = full pool.
 
     ffn_events: optional (begin, end) torch.cuda.Event pair recorded around the
     expert-FFN kernel on the launch stream.  wait_limit_ns: limit of the FFN
     kernel's bounded waits (0: 1 s).  test_starve_first_down: tests only, makes
-    the first down item's dependency wait run out.
+    the first down item's dependency wait run out.  ffn_items: form of the FFN
+    work items (0 or -1 the default, 1 CTA-pair items where the layer allows).
     """
     s, out, workspace = _prep(hidden, router_w, w_gate_up, w_down, top_k, out, workspace)
     if retained_idx is not None:
         _dev(retained_idx, torch.int32, "retained_idx")
-    opts = _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns, test_starve_first_down)
+    opts = _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns, test_starve_first_down,
+                 ffn_items)
     n_ret = 0 if retained_idx is None else int(retained_idx.numel())
     _check(load().slimwise_moe_decode_ex(
         _ptr(hidden), _ptr(router_w), _ptr(retained_idx), n_ret, _ptr(w_gate_up), _ptr(w_down),

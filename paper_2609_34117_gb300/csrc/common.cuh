@@ -195,15 +195,17 @@ struct Dims {
   int Is;         // shared-expert intermediate width (0: no shared expert)
   int S;          // shared-expert work entries: ceil(B / tok_chunk), 0 without one
   int wide;       // 1: a routed work item covers two adjacent 128-row weight tiles
+  int pair;       // 1: the same two tiles, one per CTA of a 2-CTA cluster (M = 256 MMA)
 };
 
 // Work items per entry: routed gate/up tiles (64 gate + 64 up rows each, or
 // twice that for wide items) and down tiles (128 rows of W_down, or 256).
+__host__ __device__ inline int item_tiles(const Dims &d) { return (d.wide || d.pair) ? 2 : 1; }
 __host__ __device__ inline int gate_up_tiles(const Dims &d) {
-  return d.I / (kGateRows * (d.wide ? 2 : 1));
+  return d.I / (kGateRows * item_tiles(d));
 }
 __host__ __device__ inline int down_tiles(const Dims &d) {
-  return d.H / (kTileRows * (d.wide ? 2 : 1));
+  return d.H / (kTileRows * item_tiles(d));
 }
 // Wide items need whole 256-row tiles of both weights and no shared expert
 // (its items keep 128 rows, and a stage holds one kind of A tile).  Two
@@ -217,6 +219,14 @@ __host__ __device__ inline int down_tiles(const Dims &d) {
 constexpr int kWideMinChunk = 64;
 constexpr int kWideMaxChunk = 80;
 constexpr int kWideMinPool = 64;
+// Pair items: a work item's two 128-row weight tiles go to the two CTAs of a
+// cluster, which run one M = 256 MMA (tcgen05 cta_group::2) whose N operand,
+// the token rows, is split between their shared memories.  Each CTA then
+// holds 128 weight rows and half of the token rows per stage: the token rows
+// read per weight byte halve, and a stage shrinks, so more of them fit.  On
+// the Qwen-class layer they measured slower than 128-row items at every load
+// tried (B = 64-512, m' = 32-128: 15-40 %), so a layer uses them only when
+// the caller asks (slimwise_decode_opts.ffn_items = 1).
 
 // Kernel launch declarations (defined in their own translation units).
 cudaError_t launch_route_topk(const __nv_bfloat16 *hidden, const float *router_w,
@@ -229,8 +239,10 @@ cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shar
 struct FfnMaps {
   CUtensorMap w_gu;                 // [E*2I rows, H cols] bf16, box 64 x 64
   CUtensorMap w_down;               // [E*H rows, I cols] bf16, box 64 x 64
-  CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16, box 64 x 16 (m + 1)
-  CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16, box 64 x 16 (m + 1)
+  // token rows: box 64 x 16 (m + 1), or 64 x 8 (m + 1) for pair items (each
+  // CTA of the pair loads half of an item's rows)
+  CUtensorMap xp[kTokBoxSizes];     // [B*k rows, H cols] bf16
+  CUtensorMap act[kTokBoxSizes];    // [B*k rows, I cols] bf16
   // shared expert (encoded only when there is one)
   CUtensorMap w_gu_s;               // [2Is rows, H cols] bf16, box 64 x 64
   CUtensorMap w_down_s;             // [H rows, Is cols] bf16, box 64 x 64
@@ -349,6 +361,68 @@ __device__ __forceinline__ bool mbar_wait_timeout(uint32_t bar, uint32_t parity,
   }
 }
 
+// Clusters (CTA pairs of the expert FFN) ------------------------------------
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address, in the cluster's shared window, of the variable at shared address
+// `addr` of this CTA, in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+// Arrive on an mbarrier of another CTA of the cluster (cluster address),
+// releasing this thread's earlier memory operations at cluster scope.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cl_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cl_bar)
+               : "memory");
+}
+__device__ __forceinline__ uint32_t ld_shared_cluster(uint32_t cl_addr) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(cl_addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_shared_cluster(uint32_t cl_addr, int v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cl_addr), "r"(v) : "memory");
+}
+// try_wait acquiring at cluster scope: for barriers that another CTA arrives on.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded cluster-scope wait: false after `timeout_ns`, or once *abort is set
+// (abort may be NULL: the wait then ignores it).
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity,
+                                                          volatile int *abort,
+                                                          uint64_t timeout_ns) {
+#pragma unroll 1
+  for (int i = 0; i < 256; ++i)
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+#pragma unroll 1
+  while (true) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (abort && *abort) return false;
+    if (global_timer_ns() - t0 > timeout_ns) return false;
+  }
+}
+// Every thread of every CTA of the cluster.
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile(
+      "barrier.cluster.arrive.release.aligned;\n\t"
+      "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // TMA -----------------------------------------------------------------------
 __device__ __forceinline__ void tma_prefetch_desc(const void *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
@@ -371,6 +445,18 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *map,
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_"
       "tx::bytes.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+// The same load by the second CTA of a pair: the data lands in this CTA's
+// shared memory and completes bytes on the pair leader's mbarrier
+// (`cl_bar`, a cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void *map,
+                                                 uint32_t cl_bar, int x, int y,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::"
+      "bytes.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(cl_bar), "l"(policy)
       : "memory");
 }
 // L2 prefetch of one box of a 2-D tensor map (no shared memory, no barrier).
@@ -408,6 +494,23 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
                "r"(ncols)
                : "memory");
 }
+// The CTA-pair forms (cta_group::2): alloc, relinquish and dealloc are run
+// by one warp of each CTA of the pair; every tcgen05 instruction of a kernel
+// uses one cta_group.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile(
+      "tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+      "r"(ncols)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr),
+               "r"(ncols)
+               : "memory");
+}
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -424,6 +527,29 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc,
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
           d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// M = 256 over the CTA pair (issued by the pair's first CTA): A rows 0-127
+// and D lanes 0-127 in that CTA, rows 128-255 in the second; the N operand's
+// rows are split in halves, the first half in the first CTA.  The smem
+// descriptors address both CTAs' operands at the same offsets.
+__device__ __forceinline__ void tc_mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc,
+                                                 uint64_t b_desc, uint32_t idesc,
+                                                 uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the mbarrier at shared address `bar` of each CTA in `cta_mask`
+// once every previously issued pair MMA of this thread completed.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster."
+      "b64 [%0], %1;" ::"r"(bar),
+      "h"(cta_mask)
       : "memory");
 }
 // Arrive on `bar` once every previously issued MMA of this thread completed.

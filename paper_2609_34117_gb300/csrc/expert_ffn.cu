@@ -56,7 +56,7 @@ constexpr int kXchBytes = kEpiGroups * kTileRows * kXchStride * 4;
 
 // A pipeline stage: one 64-wide K sub-tile (one 128-byte swizzle atom) of
 // the item's weight rows -- 128, or 256 for a wide item -- then tok_chunk
-// token rows of the same K range.
+// token rows of the same K range (half of them in each CTA of a pair).
 struct FfnSmem {
   int stages;
   int a_bytes;
@@ -64,17 +64,19 @@ struct FfnSmem {
   size_t xch_off, bar_off, misc_off, total;
 };
 
-__host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages, int wide) {
+__host__ __device__ inline FfnSmem ffn_smem_plan(int tok_chunk, int stages, int wide,
+                                                  int pair) {
   FfnSmem p;
   p.stages = stages;
   p.a_bytes = kATileBytes * (wide ? 2 : 1);
-  p.stage_bytes = p.a_bytes + tok_chunk * kBlockK * 2;
+  p.stage_bytes = p.a_bytes + (pair ? tok_chunk / 2 : tok_chunk) * kBlockK * 2;
   p.xch_off = (size_t)stages * p.stage_bytes;
   p.bar_off = p.xch_off + kXchBytes;
-  // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R], drain
-  p.misc_off = p.bar_off + 8 * (2 * stages + 4 + 2 * kItemRing + 1);
-  // item ring, tmem base, abort, consumed stages
-  p.total = p.misc_off + 4 * (kItemRing + 3) + 1024;
+  // full[S], empty[S], acc_full[2], acc_empty[2], item_full[R], item_empty[R],
+  // drain, and for a pair mailbox_full[R], mailbox_empty[R]
+  p.misc_off = p.bar_off + 8 * (2 * stages + 4 + 2 * kItemRing + 1 + (pair ? 2 * kItemRing : 0));
+  // item ring, tmem base, abort, consumed stages, and for a pair the mailbox[R]
+  p.total = p.misc_off + 4 * (kItemRing + 3 + (pair ? kItemRing : 0)) + 1024;
   return p;
 }
 
@@ -224,7 +226,19 @@ __device__ __forceinline__ void raise_abort(volatile int *abort, Ws &ws, int bit
 // At most 128 registers a thread (320 threads: 40 K of the SM's 64 K), so
 // that a CTA of the dependent combine kernel (256 threads, 72 registers)
 // can become resident beside this one.
-template <bool kShared, bool kWide>
+//
+// kPair: the grid is made of 2-CTA clusters.  A routed work item covers two
+// adjacent 128-row weight tiles (as a wide item does); CTA r of the pair
+// loads tile r and token rows [r N/2, (r + 1) N/2) of the item's N, and the
+// pair's first CTA issues one M = 256 MMA per K step over both CTAs' shared
+// memory.  Only that CTA's producer takes items from the global counter; it
+// hands each one to the second CTA through a mailbox in the second CTA's
+// shared memory, so both CTAs work through the same items in the same order.
+// The second CTA's copies complete bytes on the first CTA's stage barriers;
+// the MMA commits arrive on the stage and accumulator barriers of both CTAs;
+// each CTA's epilogue reads its own TMEM lanes (its 128 weight rows) and
+// releases the accumulator to the first CTA's MMA issuer.
+template <bool kShared, bool kWide, bool kPair>
 __global__ void __maxnreg__(128)
     expert_ffn_kernel(const __grid_constant__ FfnMaps maps, Dims d, Ws ws,
                       __nv_bfloat16 *__restrict__ out,
@@ -232,10 +246,11 @@ __global__ void __maxnreg__(128)
                       int tmem_cols, int static_first, int early_dependents,
                       uint64_t timeout_ns,
                       int starve_first_down) {
+  static_assert(!(kPair && (kShared || kWide)), "pair items are routed 128-row tiles");
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const FfnSmem plan = ffn_smem_plan(d.tok_chunk, stages, d.wide);
+  const FfnSmem plan = ffn_smem_plan(d.tok_chunk, stages, d.wide, kPair ? 1 : 0);
   const uint32_t smem_base = smem_u32(smem);
   float *xch = reinterpret_cast<float *>(smem + plan.xch_off);
   const uint32_t bar0 = smem_base + (uint32_t)plan.bar_off;
@@ -246,13 +261,19 @@ __global__ void __maxnreg__(128)
   auto itf_bar = [&](int r) { return bar0 + 8u * (2 * stages + 4 + r); };
   auto ite_bar = [&](int r) { return bar0 + 8u * (2 * stages + 4 + kItemRing + r); };
   const uint32_t drain_bar = bar0 + 8u * (2 * stages + 4 + 2 * kItemRing);
+  // pair mailbox: full barriers live in the second CTA, empty ones in the first
+  auto mbf_bar = [&](int r) { return bar0 + 8u * (2 * stages + 5 + 2 * kItemRing + r); };
+  auto mbe_bar = [&](int r) { return bar0 + 8u * (2 * stages + 5 + 3 * kItemRing + r); };
   int *misc = reinterpret_cast<int *>(smem + plan.misc_off);
   volatile int *ring = misc;                         // [kItemRing]
   volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(misc + kItemRing);
   volatile int *abort = misc + kItemRing + 1;
   volatile int *consumed = misc + kItemRing + 2;     // stages the MMA finished with
+  volatile int *mbox = misc + kItemRing + 3;         // [kItemRing], pair only
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t crank = kPair ? cluster_ctarank() : 0u;  // CTA of the pair
+  const bool lead = crank == 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -261,11 +282,16 @@ __global__ void __maxnreg__(128)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(accf_bar(b), 1);
-      mbar_init(acce_bar(b), kEpiThreads);
+      // a pair's accumulator is released by one thread of each CTA's group
+      mbar_init(acce_bar(b), kPair ? 2 : kEpiThreads);
     }
     for (int r = 0; r < kItemRing; ++r) {
       mbar_init(itf_bar(r), 1);
       mbar_init(ite_bar(r), 1 + kEpiGroups * kEpiThreads);
+      if constexpr (kPair) {
+        mbar_init(mbf_bar(r), 1);
+        mbar_init(mbe_bar(r), 1);
+      }
     }
     mbar_init(drain_bar, 1);
     *abort = 0;
@@ -289,35 +315,52 @@ __global__ void __maxnreg__(128)
     }
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32((const void *)tmem_slot), (uint32_t)tmem_cols);
-    tmem_relinquish();
+    if constexpr (kPair) {
+      tmem_alloc_pair(smem_u32((const void *)tmem_slot), (uint32_t)tmem_cols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_u32((const void *)tmem_slot), (uint32_t)tmem_cols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
+  // both CTAs' barriers are initialised before either arrives on the other's
+  if constexpr (kPair) cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // the pair MMA writes both CTAs' accumulators at the first CTA's address:
+  // the second CTA checks that its allocation is the same, else it takes no
+  // work (its partner's waits then run out)
+  if constexpr (kPair) {
+    if (threadIdx.x == 0 && !lead &&
+        ld_shared_cluster(mapa_shared(smem_u32((const void *)tmem_slot), 0u)) != tmem_base)
+      raise_abort(abort, ws, SLIMWISE_DEVERR_TMEM_PAIR);
+  }
 
   // While the grouping kernel runs (this grid may already be resident), warm
   // L2 with this CTA's likely first work item: the gate/up tile that item
-  // number blockIdx.x has when each retained expert is selected and takes one
-  // entry.  The work list runs in ascending expert order, so entry j is then
-  // the j-th retained expert (retained ids listed in ascending order), which
-  // holds for nearly every pool once B k >= 2 m'.  The guess uses only this
-  // call's inputs, so it is as good for a stack of different layers as for
-  // one layer called again (guessing from the previous call's work list cost
-  // a 10-layer skewed stack 3.8 %).  A wide item warms only its first 64 gate
-  // and 64 up rows: all of them would be 152 MB, more than L2 holds.
-  // Prefetches only, every index bounded, so a wrong guess costs bandwidth,
-  // never correctness.
+  // number blockIdx.x (for a pair, the cluster's number) has when each
+  // retained expert is selected and takes one entry.  The work list runs in
+  // ascending expert order, so entry j is then the j-th retained expert
+  // (retained ids listed in ascending order), which holds for nearly every
+  // pool once B k >= 2 m'.  The guess uses only this call's inputs, so it is
+  // as good for a stack of different layers as for one layer called again
+  // (guessing from the previous call's work list cost a 10-layer skewed stack
+  // 3.8 %).  A wide item warms only its first 64 gate and 64 up rows: all of
+  // them would be 152 MB, more than L2 holds; each CTA of a pair warms its
+  // own 64 gate and 64 up rows.  Prefetches only, every index bounded, so a
+  // wrong guess costs bandwidth, never correctness.
+  const int item0 = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
   if constexpr (!kShared) {
     if (warp == 0 && lane == 0 && d.B * d.k >= 2 * d.m_ret) {
       const int t1g = gate_up_tiles(d);
-      const int rows = kGateRows * (d.wide ? 2 : 1);  // gate rows (and up rows) of a tile
-      const int entry = blockIdx.x / t1g;
+      const int rows = kGateRows * item_tiles(d);  // gate rows (and up rows) of an item
+      const int entry = item0 / t1g;
       if (entry < d.m_ret) {
         const int e = retained ? __ldcg(retained + entry) : entry;
         if (e >= 0 && e < d.E) {
-          const int row0 = e * 2 * d.I + (blockIdx.x - entry * t1g) * rows;
+          const int row0 = e * 2 * d.I + (item0 - entry * t1g) * rows + (int)crank * kGateRows;
           for (int kc = 0; kc < d.H / kBlockK; ++kc) {
             tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0);
             tma_prefetch_2d(&maps.w_gu, kc * kBlockK, row0 + d.I);
@@ -349,7 +392,10 @@ __global__ void __maxnreg__(128)
   ip.t2 = t2;
   ip.S = kShared ? d.S : 0;
   const int nb_cols = ffn_acc_cols(d);  // TMEM columns per accumulator buffer
-  constexpr int wmul = kWide ? 2 : 1;   // 128-row halves of a routed item
+  constexpr int wmul = kWide ? 2 : 1;   // 128-row halves of a routed item in this CTA
+  // 128-row tiles of a routed item (across the pair): its gate/up items count
+  // as many finished tiles towards the entry's down items
+  constexpr int tiles_per_item = (kWide || kPair) ? 2 : 1;
 
 
   if (warp == 0) {
@@ -363,15 +409,38 @@ __global__ void __maxnreg__(128)
       uint32_t rphase = 0;
       int issued = 0;
       // With every CTA of the grid resident (one per SM), CTA i's first item
-      // is item i and later ones come from the counter past the grid: the
-      // first item costs no atomic round trip after the dependency wait.
+      // is item i (for pairs, cluster i's) and later ones come from the
+      // counter past the grid: the first item costs no atomic round trip after
+      // the dependency wait.
+      const int n_first = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
       bool first = static_first != 0;
       for (;;) {
-        int item = first ? (int)blockIdx.x
-                         : (static_first ? (int)gridDim.x : 0) +
-                               atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
-        first = false;
-        if (*abort) item = 0x7FFFFFFF;
+        int item;
+        if (!kPair || lead) {
+          item = first ? item0
+                       : (static_first ? n_first : 0) + atomicAdd(&ws.ctrl[kCtrlWorkCounter], 1);
+          first = false;
+          if (*abort) item = 0x7FFFFFFF;
+          if constexpr (kPair) {
+            // hand the item to the second CTA; an item past the end (or the
+            // abort sentinel) ends its loop too
+            if (!mbar_wait_cluster_bounded(mbe_bar(slot), rphase ^ 1u, nullptr, timeout_ns)) {
+              if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+              break;
+            }
+            st_shared_cluster(mapa_shared(smem_u32((const void *)(mbox + slot)), 1u), item);
+            mbar_arrive_cluster(mapa_shared(mbf_bar(slot), 1u));
+          }
+        } else {
+          // the second CTA of a pair: the item its first CTA took
+          if (!mbar_wait_cluster_bounded(mbf_bar(slot), rphase, abort, timeout_ns)) {
+            if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+            break;
+          }
+          item = mbox[slot];
+          mbar_arrive_cluster(mapa_shared(mbe_bar(slot), 0u));
+          if (*abort) item = 0x7FFFFFFF;
+        }
         if (!mbar_wait_bounded(ite_bar(slot), rphase ^ 1u, abort, timeout_ns)) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
           break;
@@ -389,10 +458,43 @@ __global__ void __maxnreg__(128)
           break;
         }
         const Item it = decode_item<kShared>(item, ip, ws);
+        // the item's token rows: one box of the tokens rounded up to 16
+        // rows (rows past the entry are loaded but not multiplied); each CTA
+        // of a pair loads half of them, from 8 n16 rows further for the second
+        const int box_m = token_box_for(it.n16);
+        const int tok_row = it.slot_base + (kPair ? (int)crank * it.n16 * (kTokBox / 2) : 0);
+        // weight rows: per 128-row half of the item, two 64-row boxes -- the
+        // gate rows and the matching up rows, or 128 consecutive down rows;
+        // a pair's CTA r loads half r
+        const int halves = (kShared && it.shared) ? 1 : wmul;
+        const int hstep = it.down ? kTileRows : kGateRows;  // row offset of half 1
+        int nk, row0, row1;
+        const void *amap;
+        const void *bmap;
+        if (kShared && it.shared) {
+          // the shared expert: its own weights, tokens in batch order
+          nk = it.down ? d.Is / kBlockK : d.H / kBlockK;
+          amap = it.down ? (const void *)&maps.w_down_s : (const void *)&maps.w_gu_s;
+          bmap = it.down ? (const void *)&maps.act_s[box_m] : (const void *)&maps.xt[box_m];
+          row0 = it.down ? it.tile * kTileRows : it.tile * kGateRows;
+          row1 = it.down ? row0 + kGateRows : row0 + d.Is;
+        } else {
+          nk = it.down ? d.I / kBlockK : d.H / kBlockK;
+          amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
+          bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
+          const int half0 = kPair ? (int)crank : 0;
+          if (it.down) {
+            row0 = it.expert * d.H + (it.tile * tiles_per_item + half0) * kTileRows;
+            row1 = row0 + kGateRows;
+          } else {
+            row0 = it.expert * 2 * d.I + (it.tile * tiles_per_item + half0) * kGateRows;
+            row1 = row0 + d.I;
+          }
+        }
         if (it.down) {
           // the entry's activations must be complete: all its gate/up tiles
           const int *done = &ws.entry_done[it.entry];
-          int need = (kShared && it.shared) ? ip.t1s : t1;
+          int need = (kShared && it.shared) ? ip.t1s : t1 * (kPair ? 2 : 1);
           // test only: the first routed down item waits for one gate/up tile
           // more than exist, so its wait runs out (the timeout path)
           if (starve_first_down && item == ip.S * ip.t1s + ip.r1) ++need;
@@ -411,37 +513,10 @@ __global__ void __maxnreg__(128)
           if (!ok) break;
           fence_proxy_async_global();
         }
-        // the item's token rows: one box of the tokens rounded up to 16
-        // rows (rows past the entry are loaded but not multiplied)
-        const int box_m = token_box_for(it.n16);
-        // weight rows: per 128-row half of the item, two 64-row boxes -- the
-        // gate rows and the matching up rows, or 128 consecutive down rows
-        const int halves = (kShared && it.shared) ? 1 : wmul;
-        const int hstep = it.down ? kTileRows : kGateRows;  // row offset of half 1
-        int nk, row0, row1;
-        const void *amap;
-        const void *bmap;
-        if (kShared && it.shared) {
-          // the shared expert: its own weights, tokens in batch order
-          nk = it.down ? d.Is / kBlockK : d.H / kBlockK;
-          amap = it.down ? (const void *)&maps.w_down_s : (const void *)&maps.w_gu_s;
-          bmap = it.down ? (const void *)&maps.act_s[box_m] : (const void *)&maps.xt[box_m];
-          row0 = it.down ? it.tile * kTileRows : it.tile * kGateRows;
-          row1 = it.down ? row0 + kGateRows : row0 + d.Is;
-        } else {
-          nk = it.down ? d.I / kBlockK : d.H / kBlockK;
-          amap = it.down ? (const void *)&maps.w_down : (const void *)&maps.w_gu;
-          bmap = it.down ? (const void *)&maps.act[box_m] : (const void *)&maps.xp[box_m];
-          if (it.down) {
-            row0 = it.expert * d.H + it.tile * kTileRows * halves;
-            row1 = row0 + kGateRows;
-          } else {
-            row0 = it.expert * 2 * d.I + it.tile * kGateRows * halves;
-            row1 = row0 + d.I;
-          }
-        }
+        // bytes the stage barrier expects: for a pair, both CTAs' copies
         const uint32_t stage_tx =
-            (uint32_t)(halves * kATileBytes + kTokBox * (box_m + 1) * kBlockK * 2);
+            kPair ? (uint32_t)(2 * kATileBytes + it.n16 * kTokBox * kBlockK * 2)
+                  : (uint32_t)(halves * kATileBytes + kTokBox * (box_m + 1) * kBlockK * 2);
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort, timeout_ns)) {
@@ -451,13 +526,21 @@ __global__ void __maxnreg__(128)
           }
           const int x = kc * kBlockK;
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
-          mbar_arrive_expect_tx(full_bar(stage), stage_tx);
-          for (int h = 0; h < halves; ++h) {
-            const uint32_t ah = a + (uint32_t)(h * kATileBytes);
-            tma_load_2d(ah, amap, full_bar(stage), x, row0 + h * hstep, pol_w);
-            tma_load_2d(ah + kATileBytes / 2, amap, full_bar(stage), x, row1 + h * hstep, pol_w);
+          if (kPair && !lead) {
+            const uint32_t lb = mapa_shared(full_bar(stage), 0u);
+            tma_load_2d_pair(a, amap, lb, x, row0, pol_w);
+            tma_load_2d_pair(a + kATileBytes / 2, amap, lb, x, row1, pol_w);
+            tma_load_2d_pair(a + (uint32_t)plan.a_bytes, bmap, lb, x, tok_row, pol_x);
+          } else {
+            mbar_arrive_expect_tx(full_bar(stage), stage_tx);
+            for (int h = 0; h < halves; ++h) {
+              const uint32_t ah = a + (uint32_t)(h * kATileBytes);
+              tma_load_2d(ah, amap, full_bar(stage), x, row0 + h * hstep, pol_w);
+              tma_load_2d(ah + kATileBytes / 2, amap, full_bar(stage), x, row1 + h * hstep,
+                          pol_w);
+            }
+            tma_load_2d(a + (uint32_t)plan.a_bytes, bmap, full_bar(stage), x, tok_row, pol_x);
           }
-          tma_load_2d(a + (uint32_t)plan.a_bytes, bmap, full_bar(stage), x, it.slot_base, pol_x);
           ++issued;
           if (++stage == stages) {
             stage = 0;
@@ -466,7 +549,16 @@ __global__ void __maxnreg__(128)
         }
         if (!ok) break;
       }
-      if (*abort) {
+      if (kPair && !lead) {
+        // The second CTA's stages complete on the first CTA's barriers; the
+        // first CTA's MMAs read them and their commits arrive here.  Wait
+        // (bounded) until every stage still in the ring has been released,
+        // so that no copy, read or arrival is left on this CTA's shared
+        // memory when it exits.
+        const int from = issued > stages ? issued - stages : 0;
+        for (int s = from; s < issued; ++s)
+          mbar_wait_timeout(empty_bar(s % stages), (uint32_t)((s / stages) & 1), 10000000ull);
+      } else if (*abort) {
         // let this CTA's copies in flight land before shared memory goes away
         for (int s = *consumed; s < issued; ++s)
           mbar_wait_timeout(full_bar(s % stages), (uint32_t)((s / stages) & 1), 10000000ull);
@@ -475,7 +567,25 @@ __global__ void __maxnreg__(128)
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    if (lane == 0 && kPair && !lead) {
+      // the second CTA of a pair issues no MMA: it only keeps its item ring
+      // moving
+      int slot = 0;
+      uint32_t rphase = 0;
+      for (;;) {
+        if (!mbar_wait_bounded(itf_bar(slot), rphase, abort, timeout_ns)) {
+          if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
+          break;
+        }
+        const int item = ring[slot];
+        mbar_arrive(ite_bar(slot));
+        if (++slot == kItemRing) {
+          slot = 0;
+          rphase ^= 1u;
+        }
+        if (item >= total) break;
+      }
+    } else if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       int slot = 0;
@@ -497,15 +607,20 @@ __global__ void __maxnreg__(128)
         const Item it = decode_item<kShared>(item, ip, ws);
         const int b = local & 1;
         const uint32_t use = (uint32_t)(local >> 1);
-        if (!mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, timeout_ns)) {
+        const bool freed =
+            kPair ? mbar_wait_cluster_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, timeout_ns)
+                  : mbar_wait_bounded(acce_bar(b), (use & 1u) ^ 1u, abort, timeout_ns);
+        if (!freed) {
           if (!*abort) raise_abort(abort, ws, SLIMWISE_DEVERR_PIPELINE_TIMEOUT);
           break;
         }
         tc_fence_after();
         // half h of the item: A = the stage's weight rows [128 h, 128 h + 128),
-        // D = columns [h tok_chunk, ...) of the buffer; B = the token rows
+        // D = columns [h tok_chunk, ...) of the buffer; B = the token rows.
+        // A pair runs one M = 256 MMA: A rows 128-255 and B rows N/2.. are the
+        // second CTA's, at the same shared-memory offsets.
         const uint32_t d_tmem = tmem_base + (uint32_t)(b * nb_cols);
-        const uint32_t idesc = idesc_bf16_f32(kTileRows, it.n16 * kTokBox);
+        const uint32_t idesc = idesc_bf16_f32(kPair ? 2 * kTileRows : kTileRows, it.n16 * kTokBox);
         const int halves = (kShared && it.shared) ? 1 : wmul;
         const int inner = (kShared && it.shared) ? d.Is : d.I;
         const int nk = it.down ? inner / kBlockK : d.H / kBlockK;
@@ -522,14 +637,22 @@ __global__ void __maxnreg__(128)
 #endif
           const uint32_t a = smem_base + (uint32_t)(stage * plan.stage_bytes);
           const uint32_t bs = a + (uint32_t)plan.a_bytes;
-          for (int h = 0; h < halves; ++h) {
-            const uint32_t as = a + (uint32_t)(h * kATileBytes);
+          if constexpr (kPair) {
 #pragma unroll
             for (int kk = 0; kk < kBlockK / 16; ++kk)
-              tc_mma_bf16(d_tmem + (uint32_t)(h * d.tok_chunk), smem_desc_sw128(as + kk * 32),
-                          smem_desc_sw128(bs + kk * 32), idesc, (kc | kk) != 0 ? 1u : 0u);
+              tc_mma_bf16_pair(d_tmem, smem_desc_sw128(a + kk * 32), smem_desc_sw128(bs + kk * 32),
+                               idesc, (kc | kk) != 0 ? 1u : 0u);
+            tc_commit_pair(empty_bar(stage), (uint16_t)3);
+          } else {
+            for (int h = 0; h < halves; ++h) {
+              const uint32_t as = a + (uint32_t)(h * kATileBytes);
+#pragma unroll
+              for (int kk = 0; kk < kBlockK / 16; ++kk)
+                tc_mma_bf16(d_tmem + (uint32_t)(h * d.tok_chunk), smem_desc_sw128(as + kk * 32),
+                            smem_desc_sw128(bs + kk * 32), idesc, (kc | kk) != 0 ? 1u : 0u);
+            }
+            tc_commit(empty_bar(stage));
           }
-          tc_commit(empty_bar(stage));
           issued_any = true;
           *consumed = ++n_consumed;
           if (++stage == stages) {
@@ -538,10 +661,12 @@ __global__ void __maxnreg__(128)
           }
         }
         if (!ok) break;
-        tc_commit(accf_bar(b));
+        if constexpr (kPair) tc_commit_pair(accf_bar(b), (uint16_t)3);
+        else tc_commit(accf_bar(b));
       }
       if (*abort && issued_any) {
-        tc_commit(drain_bar);
+        if constexpr (kPair) tc_commit_pair(drain_bar, (uint16_t)1);
+        else tc_commit(drain_bar);
         mbar_wait_timeout(drain_bar, 0, 10000000ull);
       }
     }
@@ -579,13 +704,17 @@ __global__ void __maxnreg__(128)
       if (!epi_all(g, got)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * nb_cols);
+      // 128-row tile of the item that TMEM half hh holds: half hh of a wide
+      // item, the CTA's own half of a pair item
+      const int tile0 = (kShared && it.shared) ? it.tile
+                                               : it.tile * tiles_per_item + (kPair ? (int)crank : 0);
       if (!it.down) {
         // gate rows live in TMEM lanes 0..63, the matching up rows in 64..127
         const int n_loc = et >> 3;          // token column within a 16-chunk
         const int i0 = (et & 7) * 8;        // 8 consecutive intermediate indices
         for (int hh = 0; hh < halves; ++hh) {
           // half hh of a wide item is the 64 gate + 64 up rows of tile 2 t + hh
-          const int act_col = (it.tile * halves + hh) * kGateRows + i0;
+          const int act_col = (tile0 + hh) * kGateRows + i0;
           for (int c = 0; c < it.n16; ++c) {
             uint32_t v[16];
             tmem_ld16(taddr + (uint32_t)(hh * d.tok_chunk) + c * 16, v);
@@ -620,16 +749,20 @@ __global__ void __maxnreg__(128)
           }
         }
         tc_fence_before();
-        mbar_arrive(acce_bar(b));
+        if constexpr (!kPair) mbar_arrive(acce_bar(b));
         // publish the activations to the TMA (async proxy) readers of any CTA
         fence_proxy_async_global();
         __threadfence();
         epi_bar(g);
-        if (et == 0) atomicAdd(&ws.entry_done[it.entry], 1);
+        if (et == 0) {
+          if constexpr (kPair)
+            mbar_arrive_cluster(mapa_shared(acce_bar(b), 0u));
+          atomicAdd(&ws.entry_done[it.entry], 1);
+        }
       } else {
         __nv_bfloat16 *ybase = (kShared && it.shared) ? ws.y_s : ws.y;  // token / grouped order
         for (int hh = 0; hh < halves; ++hh) {
-          const int h = (it.tile * halves + hh) * kTileRows + row;
+          const int h = (tile0 + hh) * kTileRows + row;
           for (int c = 0; c < it.n16; ++c) {
             uint32_t v[16];
             tmem_ld16(taddr + (uint32_t)(hh * d.tok_chunk) + c * 16, v);
@@ -645,13 +778,21 @@ __global__ void __maxnreg__(128)
         // the expert outputs are all a down item writes: the combine kernel
         // that follows this grid sums them
         tc_fence_before();
-        mbar_arrive(acce_bar(b));
+        if constexpr (kPair) {
+          epi_bar(g);
+          if (et == 0) mbar_arrive_cluster(mapa_shared(acce_bar(b), 0u));
+        } else {
+          mbar_arrive(acce_bar(b));
+        }
       }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  // neither CTA of a pair leaves (or frees TMEM) while the other may still
+  // use its shared memory, barriers or TMEM
+  if constexpr (kPair) cluster_sync_all();
 #ifdef SLIMWISE_TRACE
   if (threadIdx.x == 0) {
     uint64_t t = global_timer_ns();
@@ -662,7 +803,8 @@ __global__ void __maxnreg__(128)
 #endif
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, (uint32_t)tmem_cols);
+    if constexpr (kPair) tmem_dealloc_pair(tmem_base, (uint32_t)tmem_cols);
+    else tmem_dealloc(tmem_base, (uint32_t)tmem_cols);
   }
 }
 
@@ -720,10 +862,42 @@ cudaError_t launch_combine(Dims d, Ws ws, __nv_bfloat16 *out, bool pdl, cudaStre
   return cudaLaunchKernelEx(&cfg, combine_kernel<false>, d, ws, out);
 }
 
-int ffn_stages_for(int tok_chunk, int wide, size_t smem_limit) {
+int ffn_stages_for(int tok_chunk, int wide, int pair, size_t smem_limit) {
   int s = 12;
-  while (s > 2 && ffn_smem_plan(tok_chunk, s, wide).total + 1024 > smem_limit) --s;
+  while (s > 2 && ffn_smem_plan(tok_chunk, s, wide, pair).total + 1024 > smem_limit) --s;
   return s;
+}
+
+// Clusters of two FFN CTAs that can be resident at once (the pairs' SMs must
+// share a GPC), kept per device and shared-memory size.
+cudaError_t pair_clusters_resident(const void *kernel, size_t smem, int dev, int *n) {
+  thread_local int last_dev = -1;
+  thread_local size_t last_smem = 0;
+  thread_local int last_n = 0;
+  if (dev == last_dev && smem == last_smem) {
+    *n = last_n;
+    return cudaSuccess;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(kFfnThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int c = 0;
+  cudaError_t err = cudaOccupancyMaxActiveClusters(&c, kernel, &cfg);
+  if (err != cudaSuccess) return err;
+  if (c < 1) return cudaErrorInvalidConfiguration;
+  last_dev = dev;
+  last_smem = smem;
+  last_n = c;
+  *n = c;
+  return cudaSuccess;
 }
 
 cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
@@ -745,16 +919,21 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
     return cudaErrorInvalidValue;
   // the dependent combine kernel needs no shared memory: every byte the
   // block may opt into goes to pipeline stages
-  const int stages = ffn_stages_for(d.tok_chunk, d.wide, (size_t)optin);
-  const size_t smem = ffn_smem_plan(d.tok_chunk, stages, d.wide).total + 1024;
+  const int stages = ffn_stages_for(d.tok_chunk, d.wide, d.pair, (size_t)optin);
+  const size_t smem = ffn_smem_plan(d.tok_chunk, stages, d.wide, d.pair).total + 1024;
   if (smem > (size_t)optin) return cudaErrorInvalidConfiguration;
   // wide items only without a shared expert, on whole 256-row tiles, with
   // both accumulators of two buffers in the 512 TMEM columns
   if (d.wide && (d.Is > 0 || d.I % (2 * kGateRows) != 0 || d.H % (2 * kTileRows) != 0 ||
                  d.tok_chunk > 128))
     return cudaErrorInvalidValue;
-  auto kernel = d.Is > 0 ? expert_ffn_kernel<true, false>
-                         : d.wide ? expert_ffn_kernel<false, true> : expert_ffn_kernel<false, false>;
+  // pair items likewise, and never together with wide ones
+  if (d.pair && (d.wide || d.Is > 0 || d.I % (2 * kGateRows) != 0 || d.H % (2 * kTileRows) != 0))
+    return cudaErrorInvalidValue;
+  auto kernel = d.Is > 0   ? expert_ffn_kernel<true, false, false>
+                : d.pair ? expert_ffn_kernel<false, false, true>
+                : d.wide ? expert_ffn_kernel<false, true, false>
+                         : expert_ffn_kernel<false, false, false>;
   err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
   int tmem_cols = 32;
@@ -765,14 +944,35 @@ cudaError_t launch_expert_ffn(const FfnMaps &maps, Dims d, Ws ws,
   cfg.blockDim = dim3(kFfnThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   // items are assigned statically to first CTAs only if all of them are
   // resident at once (a down item may wait on another CTA's first item)
-  const int static_first = grid <= sms ? 1 : 0;
+  int resident = sms;
+  if (d.pair) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 2;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+    int clusters = 0;
+    err = pair_clusters_resident((const void *)kernel, smem, dev, &clusters);
+    if (err != cudaSuccess) return err;
+    resident = 2 * clusters;
+    // whole pairs, no more than fit at once
+    grid &= ~1;
+    if (grid > resident) grid = resident;
+    if (grid < 2) grid = 2;
+    cfg.gridDim = dim3(grid);
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  const int static_first = grid <= resident ? 1 : 0;
   const int early_dependents = d.B > 64 ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, maps, d, ws, out, retained, stages, tmem_cols,
                             static_first, early_dependents, timeout_ns, starve_first_down);

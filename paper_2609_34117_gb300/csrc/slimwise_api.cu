@@ -109,7 +109,19 @@ Dims make_dims(const slimwise_moe_shape *s, int32_t top_k, int32_t m_ret, int32_
   d.wide = (Is == 0 && d.I % (2 * kGateRows) == 0 && d.H % (2 * kTileRows) == 0 &&
             d.tok_chunk >= kWideMinChunk && d.tok_chunk <= kWideMaxChunk &&
             m_ret >= kWideMinPool) ? 1 : 0;
+  d.pair = 0;  // CTA-pair items only on request (apply_item_form)
   return d;
+}
+
+// The caller's choice of work-item form (slimwise_decode_opts.ffn_items).
+void apply_item_form(Dims *d, int32_t form) {
+  const bool can_pair = d->Is == 0 && d->I % (2 * kGateRows) == 0 && d->H % (2 * kTileRows) == 0;
+  if (form > 0 && can_pair) {
+    d->pair = 1;
+    d->wide = 0;
+  } else if (form < 0) {
+    d->pair = 0;
+  }
 }
 
 int check_workspace(const slimwise_moe_shape *s, int32_t top_k, void *ws,
@@ -166,11 +178,11 @@ struct WeightMapsKey {
 };
 struct TokenMapsKey {
   const void *xp, *act, *xt, *act_s;
-  int H, I, Is, B, tok_chunk, device;
+  int H, I, Is, B, tok_chunk, pair, device;
   uint64_t slots;
   bool operator==(const TokenMapsKey &o) const {
     return xp == o.xp && act == o.act && xt == o.xt && act_s == o.act_s && H == o.H &&
-           I == o.I && Is == o.Is && B == o.B && tok_chunk == o.tok_chunk &&
+           I == o.I && Is == o.Is && B == o.B && tok_chunk == o.tok_chunk && pair == o.pair &&
            device == o.device && slots == o.slots;
   }
 };
@@ -184,7 +196,8 @@ bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, cons
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   const WeightMapsKey kw = {w_gate_up, w_down, se.gate_up, se.down, d.E, d.H, d.I, d.Is, dev};
-  const TokenMapsKey kt = {w.xp, w.act, w.xt, w.act_s, d.H, d.I, d.Is, d.B, d.tok_chunk, dev, slots};
+  const TokenMapsKey kt = {w.xp, w.act, w.xt, w.act_s, d.H, d.I, d.Is, d.B, d.tok_chunk, d.pair,
+                          dev, slots};
   if (!(have_w && kw == last_w)) {
     have_w = false;
     if (encode_map(&cached.w_gu, w_gate_up, (uint64_t)d.E * 2 * d.I, d.H, kGateRows) ||
@@ -199,9 +212,11 @@ bool ffn_maps_for(FfnMaps *maps, const void *w_gate_up, const void *w_down, cons
   }
   if (!(have_t && kt == last_t)) {
     have_t = false;
-    // token boxes up to the chunk: an item's box covers at most chunk rows
+    // token boxes up to the chunk: an item's box covers at most chunk rows;
+    // each CTA of a pair loads half of an item's rows, so its boxes are half
+    // as high (8 (b + 1) rows for 16 (b + 1) tokens)
     for (int b = 0; b < kTokBoxSizes && kTokBox * (b + 1) <= d.tok_chunk; ++b) {
-      const uint32_t rows = (uint32_t)(kTokBox * (b + 1));
+      const uint32_t rows = (uint32_t)((d.pair ? kTokBox / 2 : kTokBox) * (b + 1));
       if (encode_map(&cached.xp[b], w.xp, slots, d.H, rows) ||
           encode_map(&cached.act[b], w.act, slots, d.I, rows))
         return false;
@@ -244,7 +259,8 @@ int decode_impl(const void *hidden, const float *router_w, const int32_t *retain
   rc = device_info(&di);
   if (rc) return rc;
 
-  const Dims d = make_dims(shape, top_k, m_ret, se.inter);
+  Dims d = make_dims(shape, top_k, m_ret, se.inter);
+  if (opts) apply_item_form(&d, opts->ffn_items);
   const Ws w = make_ws(workspace, L);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const bool pdl = !(opts && opts->disable_pdl);
