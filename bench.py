@@ -276,8 +276,13 @@ def union_sizes(sw, layer, hidden_batches, retained, k):
     return us
 
 
-def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=None):
-    """Time `steps` layer calls; returns a dict of derived numbers."""
+def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=None, soak_s=0.0):
+    """Time `steps` layer calls; returns a dict of derived numbers.
+
+    soak_s: seconds of the same layer calls run between the warm-up and the
+    timed steps (untimed), so that the clock sampler around the call sees the
+    GPU under this load for many samples even when K is small.
+    """
     shape = layer.shape
     k = shape.top_k
     batches = [synth.hidden_states(B, shape, seed_x + j, device=device) for j in range(N_BATCHES)]
@@ -294,6 +299,10 @@ def measure_point(sw, layer, B, m_prime, steps, warmup, device, seed_x, sampler=
     stream = torch.cuda.current_stream()
     run_layer_steps(sw, layer, batches, retained, k, warmup, stream, ws_buf, out, copy_for_step)
     torch.cuda.synchronize()
+    t_soak = time.perf_counter()
+    while time.perf_counter() - t_soak < soak_s:
+        run_layer_steps(sw, layer, batches, retained, k, 200, stream, ws_buf, out, copy_for_step)
+        torch.cuda.synchronize()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     t0.record(stream)
@@ -542,7 +551,8 @@ def main_gpu(args, ws, rank, local):
 
     with ClockSampler(local) as clk:
         dist_barrier(ws)
-        pt = measure_point(sw, layer, B, m_prime, args.steps, args.warmup, device, seed_x=1)
+        pt = measure_point(sw, layer, B, m_prime, args.steps, args.warmup, device, seed_x=1,
+                           soak_s=CLOCK_SOAK_S)
         dist_barrier(ws)
     tokens, secs = aggregate(ws, B * args.steps, pt["step_ms"] * 1e-3 * args.steps)
     value = tokens / secs
@@ -569,7 +579,7 @@ def main_gpu(args, ws, rank, local):
         "step_spread": "percentiles of the mean step over blocks of 10 consecutive layer calls",
         "graph": graph,
         "gpu_launches": 4 * args.steps,   # route, group, expert FFN, combine per step
-        "clocks": clk.summary(),
+        "clocks": dict(clk.summary(), soak_s=CLOCK_SOAK_S),
     }
     if FFN_ITEMS:
         result["ffn_items"] = FFN_ITEMS
@@ -596,6 +606,10 @@ PRUNED_POINTS = ("qwen_p50_b64", "qwen_p50_b256", "qwen_p75_b64")
 # form of the expert-FFN work items for the routed layers (--ffn-items; the
 # C ABI's slimwise_decode_opts.ffn_items: 0 the default, 1 CTA-pair items)
 FFN_ITEMS = 0
+
+# untimed seconds of the headline layer's calls before its timed steps, inside
+# the clock sampler's window (about 10 samples under load at any K)
+CLOCK_SOAK_S = 1.0
 
 
 def run_pruned(sw, device, peak, local, steps=4000):
