@@ -289,6 +289,23 @@ def moe_decode_shared(x_bf16, router_w, retained, w_gate_up, w_down, k, w_shared
     return {"idx": idx, "gates": gates, "shared_gate": s, "out": out}
 
 
+def compact_layer(w_gate_up: np.ndarray, w_down: np.ndarray, router_w: np.ndarray, retained):
+    """The pruned checkpoint of one layer (Sec. 3.1): the weights and router
+    rows of the retained experts K' only, in ascending original id, so that
+    top-k ties in the compact numbering still go to the lowest original id.
+
+    Returns (w_gate_up_c [m', 2I, H], w_down_c [m', H, I], router_w_c [m', H],
+    ids int32 [m']); compact expert j is original expert ids[j].  Raises on a
+    repeated or out-of-range id.
+    """
+    ids = np.sort(np.asarray(retained, np.int64).ravel())
+    E = w_gate_up.shape[0]
+    if ids.size == 0 or ids[0] < 0 or ids[-1] >= E or np.any(ids[1:] == ids[:-1]):
+        raise ValueError("retained ids must be distinct and in [0, E)")
+    return (np.ascontiguousarray(w_gate_up[ids]), np.ascontiguousarray(w_down[ids]),
+            np.ascontiguousarray(router_w[ids]), ids.astype(np.int32))
+
+
 # ---------------------------------------------------------------------------
 # Mutation support for the pin suite: compile a modified copy of the oracle
 # source and swap it in, so a test can check that the pins catch a planted

@@ -4,6 +4,7 @@ Every mutation edits a copy of the oracle's C source on the CPU (a dropped
 term, a swapped operand, a wrong sign, index or tie-break), builds it, swaps it
 in and runs the pin functions of test_oracle_pins; at least one must fail.
 """
+import numpy as np
 import pytest
 
 import oracle
@@ -85,3 +86,37 @@ def test_planted_mistake_is_caught(name):
             except (AssertionError, ValueError, IndexError):
                 failures += 1
     assert failures > 0, f"no pin caught mutation {name}"
+
+
+# The pruned-checkpoint compaction is numpy in oracle/__init__.py: its planted
+# mistakes replace the Python function.
+def _compact_unsorted(w_gate_up, w_down, router_w, retained):
+    # the retained experts kept in the caller's order, not ascending id
+    ids = np.asarray(retained, np.int64).ravel()
+    return w_gate_up[ids], w_down[ids], router_w[ids], ids.astype(np.int32)
+
+
+def _compact_down_rows_shifted(w_gate_up, w_down, router_w, retained):
+    # the down projection taken from the neighbouring retained expert
+    ids = np.sort(np.asarray(retained, np.int64).ravel())
+    return w_gate_up[ids], w_down[np.roll(ids, 1)], router_w[ids], ids.astype(np.int32)
+
+
+def _compact_router_rows_of_pool_order(w_gate_up, w_down, router_w, retained):
+    # the first m' router rows instead of the retained experts' rows
+    ids = np.sort(np.asarray(retained, np.int64).ravel())
+    return w_gate_up[ids], w_down[ids], router_w[:ids.size], ids.astype(np.int32)
+
+
+PY_MUTATIONS = {
+    "compact_unsorted": _compact_unsorted,
+    "compact_down_rows_shifted": _compact_down_rows_shifted,
+    "compact_router_rows_of_pool_order": _compact_router_rows_of_pool_order,
+}
+
+
+@pytest.mark.parametrize("name", sorted(PY_MUTATIONS))
+def test_planted_compaction_mistake_is_caught(name, monkeypatch):
+    monkeypatch.setattr(oracle, "compact_layer", PY_MUTATIONS[name])
+    with pytest.raises((AssertionError, ValueError, IndexError)):
+        pins.test_masked_router_equals_pruned_checkpoint(oracle)

@@ -156,16 +156,27 @@ def test_gates_independent_of_removed_unselected_experts(oracle_lib):
 def test_masked_router_equals_pruned_checkpoint(oracle_lib):
     shape = synth.TINY
     x, wr, w_gu, w_d = _tiny_layer(B=5)
-    retained = synth.retained_set(shape.num_experts, 8, seed=2).numpy()
+    retained = synth.retained_set(shape.num_experts, 8, seed=2, shuffle=True).numpy()
     xb, w, gu, dn = _bits(x), wr.numpy(), _bits(w_gu), _bits(w_d)
     a = oracle_lib.moe_decode(xb, w, retained, gu, dn, shape.top_k)
     # pruned checkpoint: only the retained experts and their router rows
-    rs = np.sort(retained)
-    b = oracle_lib.moe_decode(xb, np.ascontiguousarray(w[rs]), None,
-                              np.ascontiguousarray(gu[rs]), np.ascontiguousarray(dn[rs]), shape.top_k)
-    assert np.array_equal(rs[b["idx"]], a["idx"])
+    gu_c, dn_c, w_c, ids = oracle_lib.compact_layer(gu, dn, w, retained)
+    assert gu_c.shape == (8,) + gu.shape[1:] and w_c.shape == (8, w.shape[1])
+    b = oracle_lib.moe_decode(xb, w_c, None, gu_c, dn_c, shape.top_k)
+    assert np.array_equal(ids[b["idx"]], a["idx"])
     assert np.array_equal(b["gates"], a["gates"])
     assert np.array_equal(b["out"], a["out"])
+    # with every logit tied (zero router) both forms must pick the lowest
+    # original ids: the compact experts keep ascending original order
+    z0 = np.zeros_like(w)
+    a0 = oracle_lib.moe_decode(xb, z0, retained, gu, dn, shape.top_k)
+    _, _, w0_c, ids0 = oracle_lib.compact_layer(gu, dn, z0, retained)
+    b0 = oracle_lib.moe_decode(xb, w0_c, None, gu_c, dn_c, shape.top_k)
+    assert np.array_equal(ids0[b0["idx"]], a0["idx"])
+    assert np.array_equal(b0["out"], a0["out"])
+    for bad in (np.array([1, 1, 2], np.int32), np.array([0, shape.num_experts], np.int32)):
+        with pytest.raises(ValueError):
+            oracle_lib.compact_layer(gu, dn, w, bad)
 
 
 def test_full_pool_equals_unpruned(oracle_lib):
