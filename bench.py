@@ -784,8 +784,7 @@ def main_reference(args, ws, rank):
     full_shape = shape
     if wl.get("compact"):
         # the retained experts' rows only, in ascending id order
-        ids = np.sort(ret)
-        gu, dn, wr = np.ascontiguousarray(gu[ids]), np.ascontiguousarray(dn[ids]), np.ascontiguousarray(wr[ids])
+        gu, dn, wr, _ = oracle.compact_layer(gu, dn, wr, ret)
         shape = synth.LayerShape(shape.hidden, m_prime, shape.inter, shape.top_k)
         ret = None
     batches = [synth.bf16_bits(synth.hidden_states(B, shape, 1 + j)) for j in range(N_BATCHES)]

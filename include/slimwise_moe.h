@@ -281,6 +281,36 @@ int slimwise_moe_select_retained(const double *stats, int32_t num_experts,
                                  int32_t *retained_idx, void *stream);
 
 /*
+ * Compact (pruned) checkpoint of one layer (Sec. 3.1: the router mask of
+ * Eq. 2 over the full pool and a checkpoint that holds only the retained
+ * experts K' are two forms of the same layer; a PD-disaggregated decode
+ * instance keeps only the second).  Writes, for the n_retained experts of
+ * retained_idx in ascending original id (so that top-k ties in the compact
+ * numbering still go to the lowest original id):
+ *   w_gate_up_c  bf16 [m', 2I, H]   rows of w_gate_up [E, 2I, H]
+ *   w_down_c     bf16 [m', H, I]    rows of w_down [E, H, I]
+ *   router_w_c   fp32 [m', H]       rows of router_w [E, H]
+ *   ids_c        int32 [m']         original id of compact expert j
+ * The compact layer is then run with slimwise_moe_decode_full on shape
+ * {B, H, m', I}; its outputs equal the masked pool's bit for bit, and its
+ * selections map back through ids_c.
+ *   retained_idx  device int32 [n_retained], distinct ids in [0, E), any
+ *                 order; 1 <= n_retained <= E.
+ *   shape         hidden, num_experts (E) and inter of the full layer
+ *                 (num_tokens is not used).
+ * All pointers are device pointers owned by the caller, 16-byte aligned
+ * (ids_c and retained_idx 4-byte); outputs must not overlap the inputs.  Two
+ * kernel launches on `stream`, no host synchronisation.  A repeated or
+ * out-of-range id is reported on the device, not by the return code: every
+ * entry of ids_c is then -1 and nothing else is written.
+ */
+int slimwise_moe_compact_layer(const void *w_gate_up, const void *w_down,
+                               const float *router_w, const int32_t *retained_idx,
+                               int32_t n_retained, const slimwise_moe_shape *shape,
+                               void *w_gate_up_c, void *w_down_c, float *router_w_c,
+                               int32_t *ids_c, void *stream);
+
+/*
  * slimwise_moe_decode for callers that cannot allocate device memory (an
  * engine that reserved all of its memory up front, a plugin handed only its
  * inputs and outputs): the same layer, with the scratch memory taken from a

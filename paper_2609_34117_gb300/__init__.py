@@ -9,6 +9,7 @@ from .binding import (  # noqa: F401
     SlimwiseError,
     alloc_workspace,
     load,
+    slimwise_moe_compact_layer,
     slimwise_moe_decode,
     slimwise_moe_decode_ex,
     slimwise_moe_decode_full,

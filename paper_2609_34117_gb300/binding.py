@@ -35,7 +35,7 @@ EXPORTED = (
     "slimwise_moe_group", "slimwise_moe_device_status", "slimwise_moe_decode_noalloc",
     "slimwise_moe_shared_workspace_size", "slimwise_moe_decode_shared",
     "slimwise_moe_decode_shared_ex", "slimwise_moe_expert_stats", "slimwise_moe_select_retained",
-    "slimwise_moe_noalloc_device_status",
+    "slimwise_moe_noalloc_device_status", "slimwise_moe_compact_layer",
 )
 
 
@@ -92,6 +92,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                                           ctypes.POINTER(DecodeOpts)]
             lib.slimwise_moe_expert_stats.argtypes = [P, P, P, P, i32, P, P, P, SP, P, sz]
             lib.slimwise_moe_select_retained.argtypes = [P, i32, i32, i32, P, P]
+            lib.slimwise_moe_compact_layer.argtypes = [P, P, P, P, i32, SP, P, P, P, P, P]
             for name in EXPORTED[1:]:
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
@@ -257,6 +258,31 @@ def slimwise_moe_select_retained(stats, n_retained, criterion="reap", stream=Non
                                                CRITERIA[criterion], _ptr(ids), _stream(stream)),
            "slimwise_moe_select_retained")
     return ids
+
+
+def slimwise_moe_compact_layer(w_gate_up, w_down, router_w, retained_idx, stream=None):
+    """Compact checkpoint of the retained experts (Sec. 3.1), built by the
+    library's kernels: returns (w_gate_up_c [m', 2I, H], w_down_c [m', H, I],
+    router_w_c [m', H], ids_c int32 [m']) with the experts in ascending original
+    id.  Asynchronous on the stream: on a repeated or out-of-range id every
+    ids_c entry is -1 and the other outputs are left unwritten."""
+    _dev(w_gate_up, torch.bfloat16, "w_gate_up")
+    _dev(w_down, torch.bfloat16, "w_down")
+    _dev(router_w, torch.float32, "router_w")
+    _dev(retained_idx, torch.int32, "retained_idx")
+    E, two_i, H = (int(v) for v in w_gate_up.shape)
+    m = int(retained_idx.numel())
+    s = Shape(0, H, E, two_i // 2)
+    dev = w_gate_up.device
+    gu_c = torch.empty((m, two_i, H), dtype=torch.bfloat16, device=dev)
+    d_c = torch.empty((m,) + tuple(w_down.shape[1:]), dtype=torch.bfloat16, device=dev)
+    wr_c = torch.empty((m, H), dtype=torch.float32, device=dev)
+    ids_c = torch.empty(m, dtype=torch.int32, device=dev)
+    _check(load().slimwise_moe_compact_layer(_ptr(w_gate_up), _ptr(w_down), _ptr(router_w),
+                                             _ptr(retained_idx), m, ctypes.byref(s), _ptr(gu_c),
+                                             _ptr(d_c), _ptr(wr_c), _ptr(ids_c), _stream(stream)),
+           "slimwise_moe_compact_layer")
+    return gu_c, d_c, wr_c, ids_c
 
 
 def _opts(ffn_events, disable_pdl, grid_ctas, wait_limit_ns=0, test_starve_first_down=False,

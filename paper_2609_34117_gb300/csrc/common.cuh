@@ -269,6 +269,13 @@ cudaError_t launch_expert_stats(Dims d, Ws ws, double *stats, cudaStream_t strea
 cudaError_t launch_select_retained(const double *stats, int E, int m_prime, int criterion,
                                    int32_t *ids, cudaStream_t stream);
 
+// The compact checkpoint (retained experts' weights and router rows, ascending
+// original id); ids_c all -1 on a repeated or out-of-range id.
+cudaError_t launch_compact_layer(const void *w_gate_up, const void *w_down, const float *router_w,
+                                 const int32_t *retained, int m, int E, int H, int I, int sms,
+                                 void *w_gate_up_c, void *w_down_c, float *router_w_c,
+                                 int32_t *ids_c, cudaStream_t stream);
+
 #if defined(__CUDACC__)
 // ---------------------------------------------------------------------------
 // Device helpers

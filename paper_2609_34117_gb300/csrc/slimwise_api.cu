@@ -400,6 +400,35 @@ int slimwise_moe_select_retained(const double *stats, int32_t num_experts, int32
              : SLIMWISE_ERR_CUDA;
 }
 
+int slimwise_moe_compact_layer(const void *w_gate_up, const void *w_down,
+                               const float *router_w, const int32_t *retained_idx,
+                               int32_t n_retained, const slimwise_moe_shape *shape,
+                               void *w_gate_up_c, void *w_down_c, float *router_w_c,
+                               int32_t *ids_c, void *stream) {
+  if (!shape) return SLIMWISE_ERR_INVALID_ARG;
+  // the shape checks of a layer (num_tokens unused; top-1 is always valid)
+  slimwise_moe_shape s = *shape;
+  s.num_tokens = 0;
+  int rc = check_shape(&s, 1, n_retained);
+  if (rc) return rc;
+  if (!w_gate_up || !w_down || !router_w || !retained_idx || !w_gate_up_c || !w_down_c ||
+      !router_w_c || !ids_c)
+    return SLIMWISE_ERR_INVALID_ARG;
+  if (!aligned(w_gate_up, 16) || !aligned(w_down, 16) || !aligned(router_w, 16) ||
+      !aligned(w_gate_up_c, 16) || !aligned(w_down_c, 16) || !aligned(router_w_c, 16) ||
+      !aligned(retained_idx, 4) || !aligned(ids_c, 4))
+    return SLIMWISE_ERR_UNSUPPORTED_SHAPE;
+  DeviceInfo di;
+  rc = device_info(&di);
+  if (rc) return rc;
+  return launch_compact_layer(w_gate_up, w_down, router_w, retained_idx, n_retained,
+                              shape->num_experts, shape->hidden, shape->inter, di.sms,
+                              w_gate_up_c, w_down_c, router_w_c, ids_c,
+                              reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? SLIMWISE_OK
+             : SLIMWISE_ERR_CUDA;
+}
+
 int slimwise_moe_decode(const void *hidden, const float *router_w,
                         const int32_t *retained_idx, int32_t n_retained,
                         const void *w_gate_up, const void *w_down, int32_t top_k,

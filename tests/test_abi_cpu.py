@@ -170,3 +170,26 @@ def test_statistics_entry_points_validate_without_cuda(lib):
     assert lib.slimwise_moe_select_retained(P(), 16, 8, 3, P(), None) == 1
     assert lib.slimwise_moe_select_retained(None, 16, 8, 2, P(), None) == 1
     assert lib.slimwise_moe_select_retained(P(), 16, 0, 2, None, None) == 0
+
+
+def test_compact_layer_validates_without_cuda(lib):
+    P = _fake
+    s = binding.Shape(0, 256, 16, 128)
+    args = lambda **kw: [kw.get(n, P()) for n in ("gu", "dn", "wr", "ret")]
+    out = [P(), P(), P(), P()]
+    # null input or output pointers
+    assert lib.slimwise_moe_compact_layer(None, P(), P(), P(), 8, ctypes.byref(s), *out, None) == 1
+    assert lib.slimwise_moe_compact_layer(*args(), 8, ctypes.byref(s), P(), P(), P(), None, None) == 1
+    # retained count out of [1, E]; no shape
+    assert lib.slimwise_moe_compact_layer(*args(), 0, ctypes.byref(s), *out, None) == 1
+    assert lib.slimwise_moe_compact_layer(*args(), 17, ctypes.byref(s), *out, None) == 1
+    assert lib.slimwise_moe_compact_layer(*args(), 8, None, *out, None) == 1
+    # unsupported shape; misaligned weights or ids
+    bad = binding.Shape(0, 100, 16, 128)
+    assert lib.slimwise_moe_compact_layer(*args(), 8, ctypes.byref(bad), *out, None) == 2
+    assert lib.slimwise_moe_compact_layer(*args(gu=P(0x10008)), 8, ctypes.byref(s), *out, None) == 2
+    assert lib.slimwise_moe_compact_layer(*args(ret=P(0x10002)), 8, ctypes.byref(s), *out, None) == 2
+    # num_tokens is not used: with a negative one the shape error is still
+    # the one reported (every call above and here fails before any CUDA call)
+    neg = binding.Shape(-5, 100, 16, 128)
+    assert lib.slimwise_moe_compact_layer(*args(), 8, ctypes.byref(neg), *out, None) == 2

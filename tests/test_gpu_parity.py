@@ -212,6 +212,45 @@ def test_compact_checkpoint_equals_masked_pool(qwen, m_prime):
     assert np.array_equal(ids.cpu().numpy()[ref["idx"]], ref_m[0])
 
 
+@pytest.mark.parametrize("shape_name,m_prime", [("tiny", 8), ("tiny", 16), ("qwen", 64), ("qwen", 1)])
+def test_compact_layer_kernel_equals_oracle_compaction(request, shape_name, m_prime):
+    # The compaction kernels (slimwise_moe_compact_layer) against the oracle's
+    # compaction of the same host tensors: every byte of the compact weights
+    # and router rows, and the ids, in ascending original order (a shuffled
+    # retained list; all experts, reversed; one expert).
+    layer = request.getfixturevalue(shape_name)
+    E = layer.shape.num_experts
+    if m_prime == E:
+        retained = torch.arange(E - 1, -1, -1, dtype=torch.int32)
+    else:
+        retained = synth.retained_set(E, m_prime, 7, shuffle=True)
+    gu_c, d_c, wr_c, ids = sw.slimwise_moe_compact_layer(layer.d_w_gu, layer.d_w_d, layer.d_wr,
+                                                         retained.to(DEV))
+    torch.cuda.synchronize()
+    r_gu, r_d, r_wr, r_ids = oracle.compact_layer(layer.gu_bits, layer.d_bits, layer.wr.numpy(),
+                                                  retained.numpy())
+    assert np.array_equal(ids.cpu().numpy(), r_ids)
+    assert np.array_equal(synth.bf16_bits(gu_c.cpu()), r_gu)
+    assert np.array_equal(synth.bf16_bits(d_c.cpu()), r_d)
+    assert np.array_equal(wr_c.cpu().numpy().view(np.uint32), r_wr.view(np.uint32))
+
+
+def test_compact_layer_kernel_rejects_repeated_and_out_of_range_ids(tiny):
+    from paper_2609_34117_gb300 import checkpoint
+    E = tiny.shape.num_experts
+    for bad in ([3, 5, 3, 9], [0, E, 2], [-1, 4]):
+        ret = torch.tensor(bad, dtype=torch.int32, device=DEV)
+        gu_c, d_c, wr_c, ids = sw.slimwise_moe_compact_layer(tiny.d_w_gu, tiny.d_w_d, tiny.d_wr, ret)
+        torch.cuda.synchronize()
+        assert bool((ids == -1).all())
+        with pytest.raises(ValueError):
+            checkpoint.compact_layer(tiny.d_w_gu, tiny.d_w_d, tiny.d_wr, ret)
+    # and a good call on the same stream afterwards is unaffected
+    ret = synth.retained_set(E, 8, 3).to(DEV)
+    _, _, _, ids = sw.slimwise_moe_compact_layer(tiny.d_w_gu, tiny.d_w_d, tiny.d_wr, ret)
+    assert torch.equal(ids, torch.sort(ret).values)
+
+
 class SharedExpert:
     def __init__(self, layer, inter_shared, seed):
         H = layer.shape.hidden
