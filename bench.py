@@ -585,6 +585,7 @@ def main_gpu(args, ws, rank, local):
         result["ffn_items"] = FFN_ITEMS
     if not args.no_pruned:
         result["pruned"] = run_pruned(sw, device, peak, local)
+        result["compact_checkpoint"] = run_compact(sw, device, peak)
     if args.sweep:
         result["sweep"] = run_sweep(sw, sweep_layer, device, peak,
                                     cpu=rank == 0 and not args.no_cpu_baseline)
@@ -639,6 +640,39 @@ def run_pruned(sw, device, peak, local, steps=4000):
     del layer
     torch.cuda.empty_cache()
     return pts
+
+
+def run_compact(sw, device, peak, m_prime=64, calls=50):
+    """The compact checkpoint of the Qwen-class layer's m' = 64 retained experts
+    (Sec. 3.1), built by slimwise_moe_compact_layer: model preparation, not a
+    decode step.  Events around `calls` back-to-back calls (both launches of
+    each); bytes = read + write of the retained experts' weights and router
+    rows.  The result is checked against torch.index_select of the same rows."""
+    shape = synth.QWEN
+    w_gu, w_d = synth.expert_weights(shape, 0, device=device)
+    wr = synth.router_weight(shape, 0, device=device)
+    ret = synth.retained_set(shape.num_experts, m_prime, 2, shuffle=True).to(device)
+    for _ in range(3):
+        out = sw.slimwise_moe_compact_layer(w_gu, w_d, wr, ret)
+    torch.cuda.synchronize()
+    ids = torch.sort(ret.long()).values
+    exact = (torch.equal(out[0], w_gu.index_select(0, ids)) and
+             torch.equal(out[1], w_d.index_select(0, ids)) and
+             torch.equal(out[2], wr.index_select(0, ids)) and torch.equal(out[3].long(), ids))
+    del out
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(calls):
+        sw.slimwise_moe_compact_layer(w_gu, w_d, wr, ret)
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / calls
+    nbytes = 2 * m_prime * (shape.expert_bytes + shape.hidden * 4)
+    del w_gu, w_d, wr
+    torch.cuda.empty_cache()
+    return {"retained": m_prime, "calls": calls, "ms": ms, "bytes": nbytes,
+            "gbs": nbytes / (ms * 1e-3) / 1e9, "frac_of_measured": nbytes / (ms * 1e-3) / 1e9 / peak,
+            "equals_index_select": bool(exact)}
 
 
 def cpu_oracle_all_cores(w_gu_bits, w_d_bits, wr, retained, x_bits, k, tokens):
