@@ -13,7 +13,10 @@
 // Logits follow the canonical fp32 order: lane l of a warp owns elements
 // 128c + 4l + q (q = 0..3) of every 128-wide chunk c, accumulated with fused
 // multiply-adds in (c, q) order, then the 32 lane partials are combined by an
-// xor butterfly (offsets 16, 8, 4, 2, 1).  Pruned experts are never
+// xor butterfly (offsets 16, 8, 4, 2, 1).  Two tokens' sums advance together
+// in one packed fma.rn.f32x2 (two independent fp32 fused multiply-adds, each
+// rounded as fmaf), which halves the multiply-add instructions of the
+// issue-bound logit phase at large batches without changing a bit.  Pruned experts are never
 // evaluated: restricting top-k to K' is the Eq. 2 mask with tau = -inf, with
 // no separate masking pass.  Top-k is a warp-wide arg-max repeated k times on
 // (order-preserving logit bits desc, expert id asc): each lane sorts its
@@ -45,8 +48,15 @@ __device__ __forceinline__ float logit_from_order_bits(uint32_t o) {
 }
 
 // Hidden rows are staged in shared memory either as bf16 (half the space) or
-// converted once to fp32 (no per-use conversion: one 16-byte load feeds four
-// multiply-adds).  The product and the summation order are the same.
+// converted once to fp32 (no per-use conversion).  The product and the
+// summation order are the same.  With two or more tokens per cluster the
+// tokens are staged in pairs, interleaved element by element: for token pair
+// tp, 128-wide chunk c and lane l, the quads ((tp nchunks + c) 2 + half) 32
+// + l hold elements h = 128 c + 4 l + 2 half + {0, 1} as (t, h), (t + 1, h),
+// (t, h + 1), (t + 1, h + 1), so that one load gives both tokens' values of
+// two elements and consecutive lanes read consecutive quads.  A single token
+// (TB = 1) is staged as its plain row.
+// load_x4: the four consecutive staged elements from element index i.
 __device__ __forceinline__ float4 load_x4(const __nv_bfloat16 *xs, size_t i) {
   const uint2 xr = *reinterpret_cast<const uint2 *>(xs + i);
   return make_float4(__uint_as_float(xr.x << 16), __uint_as_float(xr.x & 0xFFFF0000u),
@@ -56,34 +66,77 @@ __device__ __forceinline__ float4 load_x4(const float *xs, size_t i) {
   return *reinterpret_cast<const float4 *>(xs + i);
 }
 
+// c0 = fma(a0, w, c0) and c1 = fma(a1, w, c1): two independent fused
+// multiply-adds in one packed instruction, each rounded once to nearest
+// exactly as fmaf, so two tokens' canonical sums advance together.
+__device__ __forceinline__ void ffma2_acc(float &c0, float &c1, float a0, float a1, float w) {
+  asm("{\n\t.reg .b64 ra, rw, rc;\n\t"
+      "mov.b64 ra, {%2, %3};\n\t"
+      "mov.b64 rw, {%4, %4};\n\t"
+      "mov.b64 rc, {%0, %1};\n\t"
+      "fma.rn.f32x2 rc, ra, rw, rc;\n\t"
+      "mov.b64 {%0, %1}, rc;\n\t}"
+      : "+f"(c0), "+f"(c1)
+      : "f"(a0), "f"(a1), "f"(w));
+}
+
+// Element index of quad (tp, c, half, lane) of the paired staging.
+__device__ __forceinline__ size_t pair_quad(int tp, int nchunks, int c, int half, int lane) {
+  return ((((size_t)tp * nchunks + c) * 2 + half) * 32 + lane) * 4;
+}
+
+// Chunk c of one router row (lane's four weights w) into every token's sum,
+// elements h = 128 c + 4 lane + q in q order.
 template <int TB, typename XT>
-__device__ __forceinline__ void fma_chunk(const XT *xs, int H, int col, float4 w,
+__device__ __forceinline__ void fma_chunk(const XT *xs, int nchunks, int c, int lane, float4 w,
                                           float (&p)[TB]) {
+  if constexpr (TB == 1) {
+    const float4 x = load_x4(xs, ((size_t)c * 32 + lane) * 4);
+    p[0] = fmaf(x.x, w.x, p[0]);
+    p[0] = fmaf(x.y, w.y, p[0]);
+    p[0] = fmaf(x.z, w.z, p[0]);
+    p[0] = fmaf(x.w, w.w, p[0]);
+  } else {
 #pragma unroll
-  for (int t = 0; t < TB; ++t) {
-    const float4 x = load_x4(xs, (size_t)t * H + col);
-    p[t] = fmaf(x.x, w.x, p[t]);
-    p[t] = fmaf(x.y, w.y, p[t]);
-    p[t] = fmaf(x.z, w.z, p[t]);
-    p[t] = fmaf(x.w, w.w, p[t]);
+    for (int tp = 0; tp < TB / 2; ++tp) {
+      const float4 a = load_x4(xs, pair_quad(tp, nchunks, c, 0, lane));
+      const float4 b = load_x4(xs, pair_quad(tp, nchunks, c, 1, lane));
+      ffma2_acc(p[2 * tp], p[2 * tp + 1], a.x, a.y, w.x);
+      ffma2_acc(p[2 * tp], p[2 * tp + 1], a.z, a.w, w.y);
+      ffma2_acc(p[2 * tp], p[2 * tp + 1], b.x, b.y, w.z);
+      ffma2_acc(p[2 * tp], p[2 * tp + 1], b.z, b.w, w.w);
+    }
   }
 }
 
 // Two router rows at once: each staged hidden vector feeds both rows' sums.
 template <int TB, typename XT>
-__device__ __forceinline__ void fma_chunk2(const XT *xs, int H, int col, float4 w0, float4 w1,
-                                           float (&p0)[TB], float (&p1)[TB]) {
+__device__ __forceinline__ void fma_chunk2(const XT *xs, int nchunks, int c, int lane, float4 w0,
+                                           float4 w1, float (&p0)[TB], float (&p1)[TB]) {
+  if constexpr (TB == 1) {
+    const float4 x = load_x4(xs, ((size_t)c * 32 + lane) * 4);
+    p0[0] = fmaf(x.x, w0.x, p0[0]);
+    p0[0] = fmaf(x.y, w0.y, p0[0]);
+    p0[0] = fmaf(x.z, w0.z, p0[0]);
+    p0[0] = fmaf(x.w, w0.w, p0[0]);
+    p1[0] = fmaf(x.x, w1.x, p1[0]);
+    p1[0] = fmaf(x.y, w1.y, p1[0]);
+    p1[0] = fmaf(x.z, w1.z, p1[0]);
+    p1[0] = fmaf(x.w, w1.w, p1[0]);
+  } else {
 #pragma unroll
-  for (int t = 0; t < TB; ++t) {
-    const float4 x = load_x4(xs, (size_t)t * H + col);
-    p0[t] = fmaf(x.x, w0.x, p0[t]);
-    p0[t] = fmaf(x.y, w0.y, p0[t]);
-    p0[t] = fmaf(x.z, w0.z, p0[t]);
-    p0[t] = fmaf(x.w, w0.w, p0[t]);
-    p1[t] = fmaf(x.x, w1.x, p1[t]);
-    p1[t] = fmaf(x.y, w1.y, p1[t]);
-    p1[t] = fmaf(x.z, w1.z, p1[t]);
-    p1[t] = fmaf(x.w, w1.w, p1[t]);
+    for (int tp = 0; tp < TB / 2; ++tp) {
+      const float4 a = load_x4(xs, pair_quad(tp, nchunks, c, 0, lane));
+      const float4 b = load_x4(xs, pair_quad(tp, nchunks, c, 1, lane));
+      ffma2_acc(p0[2 * tp], p0[2 * tp + 1], a.x, a.y, w0.x);
+      ffma2_acc(p0[2 * tp], p0[2 * tp + 1], a.z, a.w, w0.y);
+      ffma2_acc(p0[2 * tp], p0[2 * tp + 1], b.x, b.y, w0.z);
+      ffma2_acc(p0[2 * tp], p0[2 * tp + 1], b.z, b.w, w0.w);
+      ffma2_acc(p1[2 * tp], p1[2 * tp + 1], a.x, a.y, w1.x);
+      ffma2_acc(p1[2 * tp], p1[2 * tp + 1], a.z, a.w, w1.y);
+      ffma2_acc(p1[2 * tp], p1[2 * tp + 1], b.x, b.y, w1.z);
+      ffma2_acc(p1[2 * tp], p1[2 * tp + 1], b.z, b.w, w1.w);
+    }
   }
 }
 
@@ -201,31 +254,61 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
 
   // Hidden rows of the cluster's tokens (16-byte vectors of 8 bf16), zero
   // past the batch.  Each thread issues TB loads before storing any, so the
-  // staging costs one memory round trip per TB * 256 vectors.
+  // staging costs one memory round trip per TB * 256 vectors.  With token
+  // pairs a thread loads the same vector of both tokens of a pair and writes
+  // the four interleaved quads it covers (lanes 2 (v mod 16) and 2 (v mod 16)
+  // + 1 of chunk v / 16, both halves).
   const int vecs = H / 8;
-  for (int i0 = 0; i0 < TB * vecs; i0 += TB * kRouteThreads) {
-    uint4 raw[TB];
-#pragma unroll
-    for (int u = 0; u < TB; ++u) {
-      const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
-      const int t = i / vecs, v = i - t * vecs;
-      raw[u] = (i < TB * vecs && t < nt)
-                   ? reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v]
-                   : make_uint4(0u, 0u, 0u, 0u);
+  const int nchunks = H / 128;
+  auto hidden_vec = [&](int t, int v) {
+    return t < nt ? reinterpret_cast<const uint4 *>(hidden + (size_t)(t0 + t) * H)[v]
+                  : make_uint4(0u, 0u, 0u, 0u);
+  };
+  if constexpr (TB == 1) {
+    for (int v = threadIdx.x; v < vecs; v += kRouteThreads) {
+      const uint4 r = hidden_vec(0, v);
+      float4 *dst = reinterpret_cast<float4 *>(xs + 8 * v);
+      dst[0] = make_float4(__uint_as_float(r.x << 16), __uint_as_float(r.x & 0xFFFF0000u),
+                           __uint_as_float(r.y << 16), __uint_as_float(r.y & 0xFFFF0000u));
+      dst[1] = make_float4(__uint_as_float(r.z << 16), __uint_as_float(r.z & 0xFFFF0000u),
+                           __uint_as_float(r.w << 16), __uint_as_float(r.w & 0xFFFF0000u));
     }
+  } else {
+    constexpr int kPairsPerPass = TB / 2;  // pair-vectors per thread per pass
+    const int items = (TB / 2) * vecs;
+    for (int i0 = 0; i0 < items; i0 += kPairsPerPass * kRouteThreads) {
+      uint4 r0[kPairsPerPass], r1[kPairsPerPass];
 #pragma unroll
-    for (int u = 0; u < TB; ++u) {
-      const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
-      if (i >= TB * vecs) break;
-      const int t = i / vecs, v = i - t * vecs;
-      if constexpr (sizeof(XT) == 2) {
-        reinterpret_cast<uint4 *>(xs)[(size_t)t * vecs + v] = raw[u];
-      } else {
-        float4 *dst = reinterpret_cast<float4 *>(xs + (size_t)t * H + 8 * v);
-        dst[0] = make_float4(__uint_as_float(raw[u].x << 16), __uint_as_float(raw[u].x & 0xFFFF0000u),
-                             __uint_as_float(raw[u].y << 16), __uint_as_float(raw[u].y & 0xFFFF0000u));
-        dst[1] = make_float4(__uint_as_float(raw[u].z << 16), __uint_as_float(raw[u].z & 0xFFFF0000u),
-                             __uint_as_float(raw[u].w << 16), __uint_as_float(raw[u].w & 0xFFFF0000u));
+      for (int u = 0; u < kPairsPerPass; ++u) {
+        const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
+        const int tp = i / vecs, v = i - tp * vecs;
+        const bool in = i < items;
+        r0[u] = in ? hidden_vec(2 * tp, v) : make_uint4(0u, 0u, 0u, 0u);
+        r1[u] = in ? hidden_vec(2 * tp + 1, v) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kPairsPerPass; ++u) {
+        const int i = i0 + u * kRouteThreads + (int)threadIdx.x;
+        if (i >= items) break;
+        const int tp = i / vecs, v = i - tp * vecs;
+        const int c = v >> 4, l0 = 2 * (v & 15);
+        // words w of a vector hold elements 2w (low half) and 2w + 1 (high)
+        const uint32_t a[4] = {r0[u].x, r0[u].y, r0[u].z, r0[u].w};
+        const uint32_t b[4] = {r1[u].x, r1[u].y, r1[u].z, r1[u].w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          // elements 2w, 2w + 1: lane l0 + w / 2, half w % 2
+          const size_t q = pair_quad(tp, nchunks, c, w & 1, l0 + (w >> 1));
+          if constexpr (sizeof(XT) == 2) {
+            // (t, 2w) | (t + 1, 2w) << 16, then the same for element 2w + 1
+            *reinterpret_cast<uint2 *>(xs + q) =
+                make_uint2((a[w] & 0xFFFFu) | (b[w] << 16), (a[w] >> 16) | (b[w] & 0xFFFF0000u));
+          } else {
+            *reinterpret_cast<float4 *>(xs + q) =
+                make_float4(__uint_as_float(a[w] << 16), __uint_as_float(b[w] << 16),
+                            __uint_as_float(a[w] & 0xFFFF0000u), __uint_as_float(b[w] & 0xFFFF0000u));
+          }
+        }
       }
     }
   }
@@ -237,7 +320,6 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
   // shared-memory reads of the staged hidden rows; the sums and their order
   // are those of one row at a time.
   const int r_lo = crank * slice, r_hi = min(m, r_lo + slice);
-  const int nchunks = H / 128;
   // At 8 tokens per cluster the staged rows' shared-memory reads bound the
   // logits, so pairs pay from two rows on (1.6 us at B = 256, m' = 64); at
   // 16 tokens (fewer warps busy) they lost 2 us at B = 512, m' = 32.
@@ -261,7 +343,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
 #pragma unroll
       for (int u = 0; u < kPairChunkBatch; ++u)
         if (c0 + u < nchunks)
-          fma_chunk2<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v0[u], v1[u], p0, p1);
+          fma_chunk2<TB>(xs, nchunks, c0 + u, lane, v0[u], v1[u], p0, p1);
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1)
@@ -291,7 +373,7 @@ __global__ void __launch_bounds__(kRouteThreads, 2)
         if (c0 + u < nchunks) v[u] = __ldg(wrow + 32 * (c0 + u));
 #pragma unroll
       for (int u = 0; u < kChunkBatch; ++u)
-        if (c0 + u < nchunks) fma_chunk<TB>(xs, H, 128 * (c0 + u) + 4 * lane, v[u], p);
+        if (c0 + u < nchunks) fma_chunk<TB>(xs, nchunks, c0 + u, lane, v[u], p);
     }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1)
