@@ -170,6 +170,28 @@ def test_qwen_sweep_points(qwen, B, m_prime):
     _case(qwen, B=B, m_prime=m_prime, seed_x=1000 + B, seed_imp=2 + m_prime, sample=32)
 
 
+@pytest.mark.parametrize("B", [31, 33, 65, 151, 153, 303, 305, 319])
+@pytest.mark.parametrize("m_prime", [None, 32])
+def test_routing_at_cluster_size_boundaries(qwen, B, m_prime):
+    # Routing clusters take 1, 2, 4, 8 or 16 tokens as B grows (thresholds
+    # 32, 64, 152, 304), staged in token pairs from 2 tokens on and summed
+    # two tokens at a time with packed multiply-adds.  Batches just either
+    # side of each threshold end a cluster on an odd token, so the last pair
+    # holds one real token beside a zero row: every token's top-k ids and
+    # gates, the union and the grouping must still equal the oracle's bit for
+    # bit (routing only; the layer's outputs are covered by the other cases).
+    shape = qwen.shape
+    x = synth.hidden_states(B, shape, 2000 + B)
+    retained = None if m_prime is None else synth.retained_set(shape.num_experts, m_prime, 9)
+    route = sw.slimwise_moe_route(x.to(DEV), qwen.d_wr, None if retained is None else retained.to(DEV),
+                                  shape.top_k, shape.num_experts, shape.inter)
+    torch.cuda.synchronize()
+    idx, gates = oracle.route(oracle.router_logits(synth.bf16_bits(x), qwen.wr.numpy()),
+                              None if retained is None else retained.numpy(), shape.top_k)
+    ref = {"idx": idx, "gates": gates, "group": oracle.group_by_expert(idx, shape.num_experts)}
+    _check_route({n: t.cpu().numpy() for n, t in route.items()}, ref, shape.num_experts)
+
+
 @pytest.mark.parametrize("B,m_prime", [(64, 192), (64, 128), (256, 64), (8, 64)])
 def test_qwen36_shaped_layer(qwen36, B, m_prime):
     # 256 experts of intermediate size 512: 25 / 50 / 75 % pruning
