@@ -14,9 +14,11 @@
 //            waits for a down item's activations, and issues each stage's
 //            copies -- the 128-row weight tile (two 64-row boxes) and the
 //            item's token rows (one box, its height the token count rounded
-//            up to 16 rows).  The issuing thread's copy rate bounds
-//            the stage rate, so a stage takes three copies whatever the
-//            number of tokens, and the descriptors are chosen once per item.
+//            up to 16 rows).  Each copy costs the issuing thread about 40 ns
+//            (a streaming probe), so a stage takes three copies whatever the
+//            number of tokens and the descriptors are chosen once per item;
+//            at that count the copy rate no longer bounds the kernel (a
+//            second issuing warp for the token box changed nothing).
 //   warp 1   MMA issuer (one thread) and TMEM owner; double-buffered
 //            accumulators so the epilogue of one item overlaps the next.
 //   warps 2-9 two epilogue warpgroups; group g handles the items of
