@@ -16,8 +16,9 @@
 // xor butterfly (offsets 16, 8, 4, 2, 1).  Two tokens' sums advance together
 // in one packed fma.rn.f32x2 (two independent fp32 fused multiply-adds, each
 // rounded as fmaf), which halves the multiply-add instructions of the
-// issue-bound logit phase at large batches without changing a bit.  Pruned experts are never
-// evaluated: restricting top-k to K' is the Eq. 2 mask with tau = -inf, with
+// issue-bound logit phase at large batches without changing a bit.  Pruned
+// experts are never evaluated: restricting top-k to K' is the Eq. 2 mask
+// with tau = -inf, with
 // no separate masking pass.  Top-k is a warp-wide arg-max repeated k times on
 // (order-preserving logit bits desc, expert id asc): each lane sorts its
 // candidates once, then every round is two warp reductions over the lanes'
@@ -157,7 +158,8 @@ struct StageType<16> {
 };
 
 
-// Shared memory of one CTA: hidden rows [TB][H] (StageType), the logits of
+// Shared memory of one CTA: hidden rows (TB x H elements of StageType, in
+// token pairs from TB = 2 on; see load_x4), the logits of
 // the tokens whose top-k it runs [ceil(TB/8)][m] fp32 (written by every CTA
 // of the cluster), retained ids [m] int32.  Rows of tokens past the batch are
 // zero, so every token slot computes (and discards) a logit.
