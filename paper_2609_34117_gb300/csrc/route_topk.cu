@@ -18,11 +18,11 @@
 // rounded as fmaf), which halves the multiply-add instructions of the
 // issue-bound logit phase at large batches without changing a bit.  Pruned
 // experts are never evaluated: restricting top-k to K' is the Eq. 2 mask
-// with tau = -inf, with
-// no separate masking pass.  Top-k is a warp-wide arg-max repeated k times on
-// (order-preserving logit bits desc, expert id asc): each lane sorts its
-// candidates once, then every round is two warp reductions over the lanes'
-// current heads, so ties go to the lowest original id whatever the order of K'.
+// with tau = -inf, with no separate masking pass.  Top-k is a warp-wide
+// arg-max repeated k times on (order-preserving logit bits desc, expert id
+// asc): each lane sorts its candidates once, then every round is two warp
+// reductions over the lanes' current heads, so ties go to the lowest
+// original id whatever the order of K'.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
