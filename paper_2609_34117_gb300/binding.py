@@ -58,15 +58,18 @@ class DecodeOpts(ctypes.Structure):
 
 
 def library_path() -> str:
-    return _build.LIB_PATH
+    """The library this process loads: $SLIMWISE_LIBRARY if set (e.g. the
+    timeline-stamping build, build.TRACE_LIB_PATH), else the in-tree build."""
+    return os.environ.get("SLIMWISE_LIBRARY") or _build.LIB_PATH
 
 
 def load(path: str | None = None) -> ctypes.CDLL:
-    """Load libslimwise.so; raises if it has not been built."""
+    """Load libslimwise.so (or `path`, or $SLIMWISE_LIBRARY); raises if it has
+    not been built."""
     global _lib
     with _lock:
         if _lib is None:
-            p = path or _build.LIB_PATH
+            p = path or library_path()
             if not os.path.exists(p):
                 raise RuntimeError(f"libslimwise.so not built ({p}); run paper_2609_34117_gb300.build.build()")
             lib = ctypes.CDLL(p)
