@@ -24,7 +24,12 @@
 
 namespace slimwise {
 
-constexpr int kGroupTokens = 2;
+// Tokens per CTA: one up to 64 tokens, two above.  Fewer tokens per CTA
+// spread the grouped-row copy over more SMs (one against two: up to 1.1 us a
+// step faster at B = 8-64), but every CTA recounts the whole batch's
+// selections, and above 64 tokens the extra CTAs cost more (B = 256: 0.9 us,
+// B = 512: 2 us slower); four per CTA was slower at every size.
+inline int group_tokens_per_cta(int B) { return B <= 64 ? 1 : 2; }
 constexpr int kGroupThreads = 512;
 
 // Exclusive scan of vals[0..n) (n <= kMaxExperts) into outp[0..n], by one
@@ -50,6 +55,7 @@ __device__ int warp_exclusive_scan(const int *vals, int *outp, int n, int lane) 
   return total;
 }
 
+template <int kGroupTokens>
 __global__ void __launch_bounds__(kGroupThreads)
     group_gather_kernel(const __nv_bfloat16 *__restrict__ hidden,
                         const float *__restrict__ w_sg, Dims d, Ws ws, int do_gather) {
@@ -254,7 +260,8 @@ __global__ void __launch_bounds__(kGroupThreads)
 cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shared_gate,
                                 Dims d, Ws ws, bool pdl, bool gather, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((d.B + kGroupTokens - 1) / kGroupTokens);
+  const int tpc = group_tokens_per_cta(d.B);
+  cfg.gridDim = dim3((d.B + tpc - 1) / tpc);
   cfg.blockDim = dim3(kGroupThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
@@ -263,7 +270,10 @@ cudaError_t launch_group_gather(const __nv_bfloat16 *hidden, const float *w_shar
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, group_gather_kernel, hidden, w_shared_gate, d, ws,
+  if (tpc == 1)
+    return cudaLaunchKernelEx(&cfg, group_gather_kernel<1>, hidden, w_shared_gate, d, ws,
+                              gather ? 1 : 0);
+  return cudaLaunchKernelEx(&cfg, group_gather_kernel<2>, hidden, w_shared_gate, d, ws,
                             gather ? 1 : 0);
 }
 
