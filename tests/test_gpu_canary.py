@@ -1,5 +1,5 @@
-"""Guard bytes around every buffer the library writes (bounds checking without
-compute-sanitizer, which this GPU pool keeps closed).
+"""Guard bytes around every buffer the library writes: a bounds check that
+needs no memory-checking tool.
 
 Each call gets its workspace and its outputs as views into larger buffers
 whose leading and trailing 64 KB hold a known pattern.  A write past either
